@@ -1,0 +1,115 @@
+"""Counter-based seeded value generator shared by the oracle side and the GPU side.
+
+This module holds no arithmetic of the method; it only turns
+``(seed, stream, flat index)`` into a synthetic value, identically on the host
+(numpy, here) and on the device (``synth.cu`` in this folder).
+
+Definition
+----------
+* Raw bits: the i-th output (i = 0, 1, ...) of a SplitMix64 generator
+  (Steele, Lea & Flood, "Fast splittable pseudorandom number generators",
+  OOPSLA 2014) whose state starts at ``key(seed, stream)``:
+  ``raw(i) = mix64(key + (i + 1) * GAMMA)``.
+* ``key(seed, stream) = mix64(seed * 2**32 + stream + GAMMA)`` (the first
+  output of a SplitMix64 started at ``seed * 2**32 + stream``).
+* Approximately normal value: the four 16-bit fields of ``raw(i)`` are summed
+  (Irwin-Hall with four terms), centred and scaled to unit variance in fp32,
+  then ``value = (n * std) + mean`` with each fp32 operation rounded to
+  nearest separately (no fused multiply-add), so host and device agree bit
+  for bit.  The distribution is bounded at +-3.46 sigma; its first two
+  moments are those of N(mean, std^2).
+* bf16 storage: round-to-nearest-even of the fp32 value.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+GAMMA = np.uint64(0x9E3779B97F4A7C15)
+M1 = np.uint64(0xBF58476D1CE4E5B9)
+M2 = np.uint64(0x94D049BB133111EB)
+# 1 / sqrt(4 * (65536**2 - 1) / 12) rounded to fp32: unit variance for the
+# sum of four uniform 16-bit integers.
+IRWIN_HALL4_SCALE = np.float32(1.0 / np.sqrt(4.0 * (65536.0 ** 2 - 1.0) / 12.0))
+IRWIN_HALL4_MEAN = 131070  # 4 * 65535 / 2
+
+_S30 = np.uint64(30)
+_S27 = np.uint64(27)
+_S31 = np.uint64(31)
+
+
+def mix64(z: np.ndarray) -> np.ndarray:
+    """SplitMix64 output function on a uint64 array (wraps mod 2**64)."""
+    z = np.asarray(z, dtype=np.uint64)
+    with np.errstate(over="ignore"):
+        z = (z ^ (z >> _S30)) * M1
+        z = (z ^ (z >> _S27)) * M2
+    return z ^ (z >> _S31)
+
+
+def stream_key(seed: int, stream: int) -> np.uint64:
+    with np.errstate(over="ignore"):
+        s = np.uint64((int(seed) << 32) + int(stream)) + GAMMA
+    return mix64(np.array([s], dtype=np.uint64))[0]
+
+
+def raw_bits(seed: int, stream: int, index: np.ndarray) -> np.ndarray:
+    key = stream_key(seed, stream)
+    idx = np.asarray(index, dtype=np.uint64)
+    with np.errstate(over="ignore"):
+        return mix64(key + (idx + np.uint64(1)) * GAMMA)
+
+
+def normal_f32(seed: int, stream: int, index: np.ndarray, std: float = 1.0,
+               mean: float = 0.0) -> np.ndarray:
+    """Approximately N(mean, std^2) fp32 values at the given flat indices."""
+    z = raw_bits(seed, stream, index)
+    m16 = np.uint64(0xFFFF)
+    s = ((z & m16) + ((z >> np.uint64(16)) & m16) + ((z >> np.uint64(32)) & m16)
+         + (z >> np.uint64(48))).astype(np.int64)
+    c = (s - IRWIN_HALL4_MEAN).astype(np.float32)  # exact: |c| < 2**24
+    n = c * IRWIN_HALL4_SCALE                     # fp32, one rounding
+    v = n * np.float32(std)                         # fp32, one rounding
+    v = v + np.float32(mean)                        # fp32, one rounding
+    return v.astype(np.float32)
+
+
+def f32_to_bf16_bits(x: np.ndarray) -> np.ndarray:
+    """Round-to-nearest-even fp32 -> bf16, returned as uint16 bit patterns."""
+    u = np.ascontiguousarray(x, dtype=np.float32).view(np.uint32).astype(np.uint64)
+    nan = (u & np.uint64(0x7FFFFFFF)) > np.uint64(0x7F800000)
+    r = (u + np.uint64(0x7FFF) + ((u >> np.uint64(16)) & np.uint64(1))) >> np.uint64(16)
+    r = np.where(nan, (u >> np.uint64(16)) | np.uint64(0x40), r)
+    return r.astype(np.uint16)
+
+
+def bf16_bits_to_f32(b: np.ndarray) -> np.ndarray:
+    return (np.asarray(b, dtype=np.uint16).astype(np.uint32) << np.uint32(16)).view(np.float32)
+
+
+def values(dtype: str, seed: int, stream: int, start: int, count: int,
+           std: float = 1.0, mean: float = 0.0) -> np.ndarray:
+    """``count`` consecutive values of one stream, stored in ``dtype``.
+
+    Returns float32 for ``"f32"`` and uint16 bf16 bit patterns for ``"bf16"``.
+    """
+    idx = np.arange(start, start + count, dtype=np.uint64)
+    v = normal_f32(seed, stream, idx, std, mean)
+    if dtype == "f32":
+        return v
+    if dtype == "bf16":
+        return f32_to_bf16_bits(v)
+    raise ValueError(f"unknown dtype {dtype!r}")
+
+
+def values_at(dtype: str, seed: int, stream: int, index: np.ndarray,
+              std: float = 1.0, mean: float = 0.0) -> np.ndarray:
+    """Values of one stream at arbitrary flat indices (same as ``values``)."""
+    v = normal_f32(seed, stream, np.asarray(index, dtype=np.uint64), std, mean)
+    return v if dtype == "f32" else f32_to_bf16_bits(v)
+
+
+def to_f64(dtype: str, stored: np.ndarray) -> np.ndarray:
+    """Widen stored values (fp32, or bf16 bit patterns) to float64."""
+    if dtype == "f32":
+        return np.asarray(stored, dtype=np.float32).astype(np.float64)
+    return bf16_bits_to_f32(stored).astype(np.float64)

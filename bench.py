@@ -1,0 +1,383 @@
+"""Decode-step throughput of the WhiteMatter hot path on GB300.
+
+One step = L calls of wm_decode_attn (layer l reads channel c(l) of the
+paged k-channel cache) + one wm_kv_mix (the cross-layer KV pool for the B
+new tokens), i.e. B decoded tokens.  Prints one JSON line.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
+  python bench.py --impl reference ...   # the fp64 CPU oracle, timed on host cores
+
+Multi-GPU runs (torchrun) are data-parallel replicas: each rank decodes its
+own batch of sequences (weak scaling) with no collective on the data path;
+only the timing barrier and the max over ranks use torch.distributed.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "decode tokens/s per step (mix+channel attention) at 1 GB300; HBM GB/s vs peak"
+DEFAULT_WORKLOAD = "no_compression"
+FALLBACK_HBM_GBS = 6800.0
+
+
+# ---------------------------------------------------------------- helpers
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def measured_peak():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def kernel_source_hash() -> str:
+    h = hashlib.sha256()
+    for f in ("attn.cu", "common.cuh", "internal.h"):
+        with open(os.path.join(ROOT, "paper_2608_18486_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def ncu_traffic(workload: str):
+    """DRAM bytes per attention launch from the committed ncu summary, if it
+    was taken on the current kernel source; else None."""
+    path = os.path.join(ROOT, "profiles", "decode_attn_traffic.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        e = d.get(workload)
+        if e and e.get("kernel_hash") == kernel_source_hash():
+            return float(e["dram_bytes_per_launch"])
+    except Exception:
+        pass
+    return None
+
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons while running."""
+
+    FIELDS = ("timestamp,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id: str):
+        self.proc = None
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "50", "-i", gpu_id], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL,
+                text=True)
+        except Exception:
+            self.proc = None
+
+    def stop(self, t0: float, t1: float):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except Exception:
+            self.proc.kill()
+            return None
+        rows = []
+        for line in out.strip().splitlines():
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                ts = time.mktime(time.strptime(parts[0].split(".")[0], "%Y/%m/%d %H:%M:%S"))
+                ts += float("0." + parts[0].split(".")[1]) if "." in parts[0] else 0.0
+                rows.append((ts, float(parts[1]), float(parts[2]), parts[5:9]))
+            except Exception:
+                continue
+        if not rows:
+            return None
+        inside = [r for r in rows if t0 - 0.25 <= r[0] <= t1 + 0.05] or rows[-3:]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in inside for i, v in enumerate(r[3]) if v == "Active"})
+        return {"sm_mhz": statistics.median(r[1] for r in inside),
+                "sm_max_mhz": max(r[2] for r in inside), "reasons": reasons,
+                "samples": len(inside)}
+
+
+# ---------------------------------------------------------------- CPU oracle timing
+def oracle_step_estimate(prob, budget_s: float = 4.0, nthreads: int | None = None):
+    """Time the fp64 oracle on a bounded sample of one decode step and
+    extrapolate to a full step (L attention layers + the pool for B tokens).
+    Returns (seconds per full step, cores used, sample description)."""
+    import numpy as np
+    from oracle import oracle as O
+    w = prob.w
+    cores = nthreads or len(os.sched_getaffinity(0))
+    # attention: one layer, a prefix of the (b, hq) units, scaled by slots read
+    units_all = [(b, hq) for b in range(w.B) for hq in range(w.Hq)]
+    q = prob.host("q")[0]
+    kp = prob.host("k_pool") if prob.pool_elems() <= (1 << 28) else None
+    t_attn, slots_done, units_done = 0.0, 0, 0
+    if kp is not None:
+        vp = prob.host("v_pool")
+        step = max(1, cores)
+        i = 0
+        while i < len(units_all) and t_attn < budget_s / 2:
+            u = units_all[i:i + step]
+            t = time.perf_counter()
+            O.decode_attn(q, kp, vp, prob.page_table, prob.seq_lens, chan=prob.chan[0], Hq=w.Hq,
+                          Hkv=w.Hkv, d=w.d, P=w.page, units=u, nthreads=cores)
+            t_attn += time.perf_counter() - t
+            slots_done += sum(int(prob.seq_lens[b]) for b, _ in u)
+            units_done += len(u)
+            i += step
+    else:
+        from tests import _harness as H  # per-unit regeneration for pools too big for host RAM
+        i = 0
+        while i < len(units_all) and t_attn < budget_s / 2:
+            b, hq = units_all[i]
+            t = time.perf_counter()
+            H.oracle_attn_unit(prob, 0, b, hq)
+            t_attn += time.perf_counter() - t
+            slots_done += int(prob.seq_lens[b])
+            units_done += 1
+            i += 1
+    slots_total = int(sum(int(s) for s in prob.seq_lens)) * w.Hq
+    attn_step = w.L * t_attn * slots_total / max(slots_done, 1)
+    # the pool: whole tokens until the budget is spent
+    h = prob.host("h")
+    args = [prob.host(n) for n in ("pre_g", "Wr", "br", "ch_g", "Wkv", "qk_g")] \
+        if w.D * w.D * w.k <= (1 << 27) else None
+    t_mix, tok = 0.0, 0
+    if args is not None:
+        while tok < w.B and t_mix < budget_s / 2:
+            n = min(cores, w.B - tok)
+            pos = (prob.seq_lens[tok:tok + n] - 1).astype(np.float64)
+            t = time.perf_counter()
+            O.kv_mix(h[tok:tok + n], pos, *args, L=w.L, k=w.k, D=w.D, Hkv=w.Hkv, d=w.d, p=w.p,
+                     eps=w.eps_rms, eps_qk=w.eps_qk, theta=w.rope_theta, nthreads=cores)
+            t_mix += time.perf_counter() - t
+            tok += n
+    mix_step = t_mix * w.B / tok if tok else 0.0
+    sample = (f"layer 0 attention for {units_done} of {len(units_all)} (sequence, head) units "
+              f"({slots_done} slot reads), extrapolated by slots x {w.L} layers; pool for "
+              f"{tok} of {w.B} tokens, extrapolated by tokens")
+    return attn_step + mix_step, cores, sample
+
+
+# ---------------------------------------------------------------- arms
+def run_reference(args, w):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return
+    from wm_synth.inputs import make_problem
+    prob = make_problem(w, seed=0)
+    times = []
+    cores, sample = None, ""
+    for i in range(args.warmup + args.steps):
+        t, cores, sample = oracle_step_estimate(prob, budget_s=args.ref_budget)
+        if i >= args.warmup:
+            times.append(t)
+    step_s = statistics.median(times)
+    value = w.B / step_s
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s",
+            "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": step_s * 1e3, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": config_dict(w, world),
+            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores,
+                             "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def config_dict(w, world):
+    return {"workload": w.name, "L": w.L, "k": w.k, "D": w.D, "Hq": w.Hq, "Hkv": w.Hkv,
+            "d": w.d, "batch_per_gpu": w.B, "global_batch": w.B * world,
+            "context": w.ctx if not w.ctx_lo else f"U[{w.ctx_lo},{w.ctx}]", "page": w.page,
+            "p": w.p, "channel_map": w.chan_map,
+            "l2": "inputs larger than L2: each step reads every channel once (> 129 MB)",
+            "parallelism": f"replicas x{world} (batch-sharded, no collective)"}
+
+
+def run_gpu(args, w):
+    import numpy as np
+    import torch
+    import torch.distributed as dist
+
+    rank, world, local = dist_env()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1 and not dist.is_initialized():
+        dist.init_process_group("nccl", device_id=dev)
+
+    from paper_2608_18486_gb300 import make_config
+    from paper_2608_18486_gb300.session import DecodeSession
+    from wm_synth import configs as C
+    from wm_synth.device_problem import DeviceProblem
+    from wm_synth.inputs import make_problem
+
+    prob = make_problem(w, seed=rank)  # each replica decodes its own sequences
+    cfg = make_config(w.L, w.k, w.D, w.Hq, w.Hkv, w.d, w.p, w.page, w.dtype, w.chan_of_layer(),
+                      w.eps_rms, w.eps_qk, w.rope_theta)
+    sess = DecodeSession(cfg, w.B, prob.num_pages, prob.max_pages, dev)
+    dp = DeviceProblem(prob, sess.k_pool, sess.v_pool, dev)
+    sess.set_weights(*dp.weights())
+    stream = torch.cuda.Stream(dev)
+    outs = torch.empty((w.L, w.B, w.Hq, w.d), dtype=sess.dtype, device=dev)
+    torch.cuda.synchronize()
+
+    def step(ev_attn=None):
+        if ev_attn is not None:
+            ev_attn[0].record(stream)
+        for layer in range(w.L):
+            sess.decode_attn(layer, dp.q[layer], dp.page_table, dp.seq_lens, outs[layer],
+                             stream=stream)
+        if ev_attn is not None:
+            ev_attn[1].record(stream)
+        sess.kv_mix(dp.h, dp.page_table, dp.slot, stream=stream)
+
+    def barrier():
+        torch.cuda.synchronize(dev)
+        if world > 1:
+            dist.barrier()
+
+    with torch.cuda.stream(stream):
+        for _ in range(args.warmup):
+            step()
+    barrier()
+    if sess.read_status() != 0:
+        raise RuntimeError("device status set during warm-up")
+
+    gpu_uuid = str(getattr(torch.cuda.get_device_properties(dev), "uuid", "") or local)
+    if gpu_uuid and not gpu_uuid.startswith("GPU-") and len(gpu_uuid) > 8:
+        gpu_uuid = "GPU-" + gpu_uuid
+    sampler = ClockSampler(gpu_uuid) if rank == 0 else None
+    time.sleep(0.3 if sampler else 0)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier()
+    t0 = time.time()
+    start.record(stream)
+    with torch.cuda.stream(stream):
+        for i in range(args.steps):
+            step(ev[i])
+    end.record(stream)
+    barrier()
+    t1 = time.time()
+    clocks = sampler.stop(t0, t1) if sampler else None
+    status = sess.read_status()
+    if status != 0:
+        raise RuntimeError(f"device status {status} during the timed region")
+    ms = start.elapsed_time(end)
+    attn_ms = sum(a.elapsed_time(b) for a, b in ev)
+    t = torch.tensor([ms, attn_ms], dtype=torch.float64, device=dev)
+    if world > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    ms, attn_ms = float(t[0]), float(t[1])
+
+    # ---- end to end through the public API with pinned host buffers
+    q_host = torch.empty(dp.q.shape, dtype=dp.q.dtype, pin_memory=True)
+    q_host.copy_(dp.q)
+    h_host = torch.empty(dp.h.shape, dtype=dp.h.dtype, pin_memory=True)
+    h_host.copy_(dp.h)
+    out_host = torch.empty(outs.shape, dtype=outs.dtype, pin_memory=True)
+    e2e_steps = max(1, args.steps)
+
+    def e2e_step():
+        dp.q.copy_(q_host, non_blocking=True)
+        dp.h.copy_(h_host, non_blocking=True)
+        step()
+        out_host.copy_(outs, non_blocking=True)
+
+    with torch.cuda.stream(stream):
+        e2e_step()
+    barrier()
+    e_start, e_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e_start.record(stream)
+    with torch.cuda.stream(stream):
+        for _ in range(e2e_steps):
+            e2e_step()
+    e_end.record(stream)
+    barrier()
+    e2e_ms = e_start.elapsed_time(e_end)
+    te = torch.tensor([e2e_ms], dtype=torch.float64, device=dev)
+    if world > 1:
+        dist.all_reduce(te, op=dist.ReduceOp.MAX)
+    e2e_ms = float(te[0])
+
+    if rank == 0:
+        tokens = w.B * world * args.steps
+        value = tokens / (ms / 1e3)
+        launch_bytes = C.attn_launch_bytes(w, prob.seq_lens)
+        attn_launch_s = attn_ms / 1e3 / (args.steps * w.L)
+        achieved = launch_bytes / attn_launch_s / 1e9
+        peak, peak_kind = measured_peak()
+        traffic = ncu_traffic(w.name)
+        step_bytes = C.step_bytes(w, prob.seq_lens)
+        cpu_s, cores, sample = oracle_step_estimate(prob, budget_s=args.ref_budget)
+        line = {
+            "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": w.dtype,
+            "data": "synthetic", "config": config_dict(w, world),
+            "roofline": {"bound": "hbm", "kernel": "decode_attn_kernel", "achieved": achieved,
+                         "peak": peak, "peak_kind": peak_kind, "unit": "GB/s",
+                         "frac": achieved / peak, "traffic": traffic,
+                         "algorithmic_bytes_per_launch": launch_bytes,
+                         "avg_launch_us": attn_launch_s * 1e6},
+            "step_hbm_gbs": step_bytes / (ms / 1e3 / args.steps) / 1e9,
+            "attn_share_of_step": attn_ms / ms,
+            "cpu_baseline": {"value": w.B / cpu_s, "unit": "tokens/s", "cores": cores,
+                             "kind": "oracle", "sample": sample},
+            "e2e": {"value": w.B * world * e2e_steps / (e2e_ms / 1e3), "unit": "tokens/s",
+                    "h2d_bytes_per_step": int(dp.q.numel() * dp.q.element_size()
+                                              + dp.h.numel() * dp.h.element_size()),
+                    "d2h_bytes_per_step": int(outs.numel() * outs.element_size())},
+            "clocks": clocks,
+            "gpu_launches": args.steps * (w.L + 5),
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.barrier()
+        dist.destroy_process_group()
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
+    ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
+    ap.add_argument("--ref-budget", type=float, default=4.0,
+                    help="seconds of oracle time per reference/CPU-baseline sample")
+    args = ap.parse_args()
+    from wm_synth import configs
+    w = configs.get(args.workload)
+    if args.warmup < 3 and args.impl != "reference":
+        args.warmup = 3
+    if args.impl == "reference":
+        run_reference(args, w)
+    else:
+        run_gpu(args, w)
+
+
+if __name__ == "__main__":
+    main()

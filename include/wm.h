@@ -1,0 +1,188 @@
+/*
+ * wm.h -- C ABI of the WhiteMatter decode hot path on GB300 (sm_103a).
+ *
+ * WhiteMatter (Zhang & Ren, "All-to-All Cross-Layer Connections via KV
+ * Mixing") replaces the L per-layer KV projections of a decoder with a
+ * cross-layer KV pool (Sec. 3.1): for every token a router mixes the L layer
+ * states into k <= L channels, each channel is projected to keys and values
+ * and stored in a k-channel cache, and layer l attends over channel c(l).
+ * One decode step (Sec. 3.2) is L calls of wm_decode_attn (one per layer,
+ * each reading the existing cache) followed by one wm_kv_mix that appends
+ * the new token's channels.
+ *
+ * Conventions for every entry point:
+ *  - Memory: the caller owns and allocates everything (weights, states,
+ *    queries, outputs, cache pools, page tables, workspaces, status word).
+ *    Pointers marked "device" must be device (or managed) memory of the
+ *    current CUDA device.  The library allocates no memory and keeps no state
+ *    between calls other than a per-device attribute cache.
+ *  - Streams: `stream` is a cudaStream_t (NULL = legacy default stream).
+ *    Compute calls only enqueue work and return; results are valid after the
+ *    stream is synchronised.
+ *  - Errors: argument errors detectable on the host return synchronously
+ *    without launching anything.  A failed launch returns WM_ERR_CUDA.
+ *    Errors found by a kernel (an out-of-range page id, slot or length; a
+ *    pipeline wait that ran out) are written to the device word `dev_status`
+ *    (if not NULL) as the largest wm_status code seen, and the offending
+ *    access is skipped; no kernel traps.  The caller zeroes dev_status and
+ *    reads it after synchronising.
+ *  - dtype: WM_DT_BF16 tensors hold bf16 values (norms, router, mix and
+ *    softmax run in fp32, projections take bf16 operands with fp32
+ *    accumulation, cache and outputs are rounded to bf16); WM_DT_F32 tensors
+ *    are fp32 and every step runs in fp32 FMA arithmetic.
+ *  - Gains, router biases and weights have the dtype of the config.
+ *
+ * Cache layout (per pool, K and V alike), element (c, page, h, s, e) at
+ *   (((c * num_pages + page) * Hkv + h) * page_size + s) * d + e
+ * for channel c < k, physical page < num_pages, kv head h < Hkv, slot in page
+ * s < page_size, element e < d.  Logical slot t of sequence b lives in page
+ * page_table[b * max_pages + t / page_size] at in-page slot t % page_size.
+ * Slot 0 of every sequence holds the learned dummy KV (Sec. 3.2); the token
+ * at position i is stored at slot i + 1.  The page table is shared by all k
+ * channels.
+ */
+#ifndef WM_H_
+#define WM_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define WM_MAX_L 128
+
+typedef enum {
+  WM_OK = 0,
+  WM_ERR_INVALID_ARG = 1, /* bad pointer, size or configuration value        */
+  WM_ERR_UNSUPPORTED = 2, /* valid per the paper, not built here (e.g. d=96) */
+  WM_ERR_CUDA = 3,        /* a CUDA runtime call or launch failed            */
+  WM_ERR_BOUNDS = 4,      /* device: page id, slot or length out of range    */
+  WM_ERR_TIMEOUT = 5      /* device: a bounded pipeline wait ran out         */
+} wm_status;
+
+typedef enum { WM_DT_F32 = 0, WM_DT_BF16 = 1 } wm_dtype;
+
+/* Model shape of the pool (Sec. 3.1) and of the attention that reads it. */
+typedef struct {
+  int32_t L;          /* decoder layers = source states per token, 1..WM_MAX_L     */
+  int32_t k;          /* KV channels, 1 <= k <= L                                  */
+  int32_t D;          /* hidden width; multiple of 8, at most 4096                 */
+  int32_t Hq;         /* query heads; multiple of Hkv, Hq/Hkv in {1,2,4,8}         */
+  int32_t Hkv;        /* key/value heads per channel                               */
+  int32_t d;          /* head dimension: 64 or 128                                 */
+  int32_t p;          /* router reads every p-th layer from L-1 down, p >= 1       */
+  int32_t page_size;  /* cache slots per page: a power of two, 1..4096             */
+  int32_t dtype;      /* wm_dtype                                                  */
+  float eps_rms;      /* epsilon of the pre-mix and per-channel RMSNorms           */
+  float eps_qk;       /* epsilon of the per-channel key norm (QK-norm)             */
+  double rope_theta;  /* RoPE base: inverse frequency theta^(-2i/d), i < d/2       */
+  int32_t chan_of_layer[WM_MAX_L]; /* c(l) in [0, k): channel read by layer l     */
+} wm_config;
+
+/* Views of the two cache pools inside one caller buffer (see wm_cache_alloc). */
+typedef struct {
+  void* k_pool;       /* device: [k][num_pages][Hkv][page_size][d] rotated keys    */
+  void* v_pool;       /* device: same layout, raw values                           */
+  int32_t num_pages;  /* physical pages per channel                                */
+  int32_t k, Hkv, page_size, d, dtype; /* copied from the config, checked per call */
+} wm_cache;
+
+/* Pool parameters (Sec. 3.1 Steps 1-2); index [X] is the branch, 0 = K, 1 = V.
+ * All device pointers, dtype of the config, row-major:
+ *   pre_g[X] [D]                pre-mix RMSNorm gain of branch X
+ *   Wr[X]    [k*L][Lp*D]        router weights, Lp = ceil(L/p); input block m
+ *                               holds the normed state of layer L-1-m*p
+ *   br[X]    [k*L]              router bias; output j*L+l is alpha[j][l]
+ *   ch_g[X]  [k][D]             per-channel RMSNorm gains
+ *   Wkv[X]   [k][Hkv*d][D]      per-channel projections W^K_j / W^V_j
+ *   qk_g     [k][d]             per-channel key-norm gains                    */
+typedef struct {
+  const void* pre_g[2];
+  const void* Wr[2];
+  const void* br[2];
+  const void* ch_g[2];
+  const void* Wkv[2];
+  const void* qk_g;
+} wm_mix_weights;
+
+/* Human-readable name of a status code (static storage). */
+const char* wm_status_string(wm_status s);
+
+/* Validate a configuration without touching the GPU.  Returns WM_OK,
+ * WM_ERR_INVALID_ARG (values outside the paper's definitions, e.g. k > L or
+ * c(l) >= k) or WM_ERR_UNSUPPORTED (shapes this library does not build). */
+wm_status wm_config_check(const wm_config* cfg);
+
+/* Bytes of device memory wm_cache_alloc needs for `num_pages` pages per
+ * channel: two pools of k*num_pages*Hkv*page_size*d elements (the k-channel
+ * cache of Sec. 3.1 Step 2: k/L of a per-layer cache), each 256-byte aligned.
+ * Returns 0 for an invalid config or num_pages < 1. */
+size_t wm_cache_bytes(const wm_config* cfg, int32_t num_pages);
+
+/* Lay the two pools out inside a caller buffer.  dev_buf must be 256-byte
+ * aligned device memory of at least wm_cache_bytes(cfg, num_pages) bytes;
+ * nothing is written to it.  Fills *out.  Errors: WM_ERR_INVALID_ARG for a
+ * NULL pointer, a misaligned or too small buffer, or a bad config. */
+wm_status wm_cache_alloc(const wm_config* cfg, void* dev_buf, size_t bytes, int32_t num_pages,
+                         wm_cache* out);
+
+/* Workspace bytes wm_kv_mix needs for a batch of B tokens. */
+size_t wm_kv_mix_workspace(const wm_config* cfg, int32_t B);
+
+/*
+ * The cross-layer KV pool for B tokens (Sec. 3.1 Steps 1-2, appended as in
+ * Sec. 3.2).  For each token b and branch X:
+ *   hhat_l   = RMSNorm_pre^X(h[b][l])                     for l < L
+ *   xi       = [hhat_{L-1}, hhat_{L-1-p}, ...]            (Lp states)
+ *   alpha    = reshape_{k x L}(Wr[X] xi + br[X])          (signed, no softmax)
+ *   htilde_j = sum_l alpha[j][l] hhat_l                   for j < k
+ *   K_j = W^K_j RMSNorm^K_j(htilde^K_j),  V_j = W^V_j RMSNorm^V_j(htilde^V_j)
+ *   Ktilde_j = RoPE(QKNorm_j(K_j) per head; pos = slot[b] - 1)
+ * and writes Ktilde_j, V_j of every channel j and kv head to logical slot
+ * slot[b] of sequence b.
+ *   h          device [B][L][D]: states entering layers 0..L-1
+ *   page_table device int32 [B][max_pages]
+ *   slot       device int32 [B]: write slot, 1 <= slot[b] < max_pages*page_size
+ *   workspace  device, >= wm_kv_mix_workspace(cfg, B) bytes, 256-byte aligned,
+ *              no contents required
+ * Only the B*k*2*Hkv*d cache elements addressed are written.  A bad slot or
+ * page id skips that token's write and sets WM_ERR_BOUNDS.  B = 0 is a no-op.
+ */
+wm_status wm_kv_mix(const wm_config* cfg, const wm_cache* cache, const wm_mix_weights* w,
+                    const void* h, const int32_t* page_table, const int32_t* slot, int32_t B,
+                    int32_t max_pages, void* workspace, size_t ws_bytes, int32_t* dev_status,
+                    void* stream);
+
+/* Workspace bytes wm_decode_attn needs for B sequences whose page tables
+ * have max_pages entries. */
+size_t wm_decode_attn_workspace(const wm_config* cfg, int32_t B, int32_t max_pages);
+
+/*
+ * Decode attention of one layer (Sec. 3.1 Step 3, with the dummy slot of
+ * Sec. 3.2): query head hq of sequence b attends over logical slots
+ * 0..seq_lens[b]-1 of channel c(layer) = cfg->chan_of_layer[layer], kv head
+ * hq / (Hq/Hkv):  out = softmax(q K^T / sqrt(d)) V, fp32 softmax and
+ * accumulation.  Slots at or beyond seq_lens[b] are never read into the
+ * result (they may hold anything, NaN included).
+ *   q          device [B][Hq][d], already normed and rotated by the caller
+ *   seq_lens   device int32 [B], 1 <= seq_lens[b] <= max_pages*page_size
+ *   out        device [B][Hq][d]
+ *   workspace  device, >= wm_decode_attn_workspace(cfg, B, max_pages) bytes,
+ *              256-byte aligned.  It must be zero-filled before its first
+ *              use; every call leaves it ready for the next one.  Calls that
+ *              share a workspace must not overlap on the GPU.
+ * A bad length or page id zero-fills that output row (length) or skips the
+ * page, and sets WM_ERR_BOUNDS.  B = 0 is a no-op.
+ */
+wm_status wm_decode_attn(const wm_config* cfg, const wm_cache* cache, int32_t layer,
+                         const void* q, const int32_t* page_table, const int32_t* seq_lens,
+                         int32_t B, int32_t max_pages, void* out, void* workspace,
+                         size_t ws_bytes, int32_t* dev_status, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* WM_H_ */

@@ -1,0 +1,72 @@
+// Launch interfaces between the C-ABI layer (wm_api.cu) and the kernels.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "wm.h"
+
+namespace wm {
+
+// ------------------------------------------------------------ attention
+struct AttnParams {
+  const void* k_pool;     // channel c(layer) base of the K pool
+  const void* v_pool;     // channel c(layer) base of the V pool
+  const void* q;          // [B][Hq][d]
+  void* out;              // [B][Hq][d]
+  const int32_t* page_table;
+  const int32_t* seq_lens;
+  float* part_o;          // [B*Hq][max_chunks][d]
+  float* part_ml;         // [B*Hq][max_chunks][2] (max, sum) in log2 units
+  int32_t* counters;      // [B*Hkv] arrival tickets, zero between launches
+  int32_t* status;
+  int64_t page_stride;    // elements between consecutive physical pages
+  int32_t Hq, Hkv, P, log2P, num_pages, max_pages, chunk_slots, max_chunks;
+  float qscale;           // log2(e) / sqrt(d)
+};
+
+int attn_stage_slots(int dtype, int d);
+cudaError_t launch_decode_attn(const AttnParams& p, int dtype, int d, int G, int B, int Hkv,
+                               cudaStream_t s);
+
+// ------------------------------------------------------------ KV pool (mix)
+constexpr int kMaxRopeHalf = 64;  // d/2 for d <= 128
+
+struct MixParams {
+  // shape
+  int32_t B, L, k, D, Hkv, d, p, Lp, P, log2P, num_pages, max_pages;
+  float eps_rms, eps_qk;
+  // inputs
+  const void* h;                  // [B][L][D]
+  const void* pre_g[2];
+  const void* Wr[2];
+  const void* br[2];
+  const void* ch_g[2];
+  const void* Wkv[2];
+  const void* qk_g;
+  const int32_t* page_table;
+  const int32_t* slot;
+  // cache
+  void* k_pool;
+  void* v_pool;
+  // workspace
+  float* inv_rms;                 // [B][L]
+  float* xi;                      // [2][B][Lp*D] router inputs (fp32)
+  float* zpart;                   // [2][nsplit_r][B][k*L] router partial sums
+  float* rope_cs;                 // [B][d/2][2] cos, sin at pos = slot - 1
+  void* xop;                      // [2][k][B][D] normed channels, dtype
+  float* proj;                    // [2][k][B][Hkv*d] projection outputs
+  int32_t nsplit_r;
+  int32_t* status;
+  double inv_freq[kMaxRopeHalf];  // theta^(-2i/d), computed on the host in fp64
+};
+
+struct MixWorkspace {
+  size_t inv_rms, xi, zpart, rope_cs, xop, proj, total;
+  int32_t nsplit_r;
+};
+
+MixWorkspace mix_workspace_layout(const wm_config& cfg, int32_t B, int sm_count);
+cudaError_t launch_kv_mix(MixParams& p, int dtype, cudaStream_t s);
+
+}  // namespace wm

@@ -1,0 +1,364 @@
+// The cross-layer KV pool for a decode batch (Sec. 3.1 Steps 1-2), appended
+// to the paged cache (Sec. 3.2).
+//
+// Kernels, in launch order:
+//   1. prenorm   : per (token, layer) inverse RMS of h_l; writes the router
+//                  input xi = [hhat_{L-1}, hhat_{L-1-p}, ...] for both branches;
+//                  per token the RoPE cos/sin at pos = slot - 1.
+//   2. router    : z = Wr[X] xi (split over the L'D reduction), fp32.
+//   3. mix       : alpha = reshape(z + br), htilde_j = sum_l alpha[j][l] hhat_l,
+//                  RMSNorm_j, rounded to the projection operand dtype.
+//   4. projection: W^X_j x^X_j for every branch and channel.
+//   5. epilogue  : keys: per-head QK-norm then RoPE; keys and values are
+//                  rounded and written to the token's cache slot.
+#include <math.h>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace wm {
+
+namespace {
+
+constexpr int kMixThreads = 256;
+constexpr int kMaxEPT = 16;   // D <= 4096 elements per block of 256 threads
+constexpr int kChanGroup = 4; // channels mixed per CTA
+
+// ---------------------------------------------------------------- prenorm
+template <typename T>
+__global__ void __launch_bounds__(kMixThreads) prenorm_kernel(const MixParams p) {
+  __shared__ float red[32];
+  __shared__ float s_r;
+  const int l = blockIdx.x, b = blockIdx.y, tid = threadIdx.x;
+  const T* hp = reinterpret_cast<const T*>(p.h) + ((int64_t)b * p.L + l) * p.D;
+  float ss = 0.f;
+  for (int e = tid; e < p.D; e += kMixThreads) {
+    const float v = ldf(hp + e);
+    ss = fmaf(v, v, ss);
+  }
+  ss = block_sum(ss, red);
+  if (tid == 0) {
+    s_r = rsqrtf(ss / (float)p.D + p.eps_rms);
+    p.inv_rms[b * p.L + l] = s_r;
+  }
+  __syncthreads();
+  const float r = s_r;
+  // router input block m holds layer L-1-m*p
+  const int from_top = p.L - 1 - l;
+  if (from_top % p.p == 0) {
+    const int m = from_top / p.p;
+    for (int X = 0; X < 2; ++X) {
+      const T* g = reinterpret_cast<const T*>(p.pre_g[X]);
+      float* xo = p.xi + ((int64_t)X * p.B + b) * ((int64_t)p.Lp * p.D) + (int64_t)m * p.D;
+      for (int e = tid; e < p.D; e += kMixThreads) xo[e] = ldf(hp + e) * r * ldf(g + e);
+    }
+  }
+  if (l == 0) {
+    // RoPE angle pos * theta^(-2i/d) in fp64, reduced to [-pi, pi] before sincosf
+    const int s = p.slot[b];
+    const double pos = (double)(s - 1);
+    for (int i = tid; i < p.d / 2; i += kMixThreads) {
+      const double a = pos * p.inv_freq[i];
+      const double two_pi = 6.283185307179586476925286766559;
+      const float ar = (float)(a - two_pi * rint(a / two_pi));
+      float sn, cs;
+      sincosf(ar, &sn, &cs);
+      p.rope_cs[((int64_t)b * (p.d / 2) + i) * 2] = cs;
+      p.rope_cs[((int64_t)b * (p.d / 2) + i) * 2 + 1] = sn;
+    }
+  }
+}
+
+// ---------------------------------------------------------------- W x^T (SIMT)
+// out[z][n][m] = sum_{k in split} W[m][k] * X[n][k], z = batch * nsplit + split.
+// Weights of batch item `bi` start at W[bi / per_branch] + (bi % per_branch) * w_stride.
+constexpr int BM = 64, BN = 32, BK = 32;
+
+struct GemmArgs {
+  const void* W[2];
+  int64_t w_stride;      // elements between consecutive items of one branch
+  int per_branch;        // batch items per branch
+  const void* X;         // [batch][N][K]
+  int64_t x_stride;      // elements between batch items of X
+  float* out;            // [batch][nsplit][N][M]
+  int M, N, K, nsplit, k_per_split;
+};
+
+template <typename T>
+__device__ __forceinline__ void load8(const T* src, float* f);
+template <>
+__device__ __forceinline__ void load8<float>(const float* src, float* f) {
+  const float4 a = *reinterpret_cast<const float4*>(src);
+  const float4 c = *reinterpret_cast<const float4*>(src + 4);
+  f[0] = a.x; f[1] = a.y; f[2] = a.z; f[3] = a.w;
+  f[4] = c.x; f[5] = c.y; f[6] = c.z; f[7] = c.w;
+}
+template <>
+__device__ __forceinline__ void load8<__nv_bfloat16>(const __nv_bfloat16* src, float* f) {
+  Elem<__nv_bfloat16>::unpack(*reinterpret_cast<const uint4*>(src), f);
+}
+
+template <typename TW, typename TX>
+__global__ void __launch_bounds__(256) gemm_wxT_simt(const GemmArgs a) {
+  __shared__ float Ws[BK][BM + 4];
+  __shared__ float Xs[BK][BN + 4];
+  const int split = blockIdx.z % a.nsplit, bi = blockIdx.z / a.nsplit;
+  const int m0 = blockIdx.x * BM, n0 = blockIdx.y * BN;
+  const int kbeg = split * a.k_per_split;
+  const int kend = min(a.K, kbeg + a.k_per_split);
+  const TW* W = reinterpret_cast<const TW*>(a.W[bi / a.per_branch]) +
+                (int64_t)(bi % a.per_branch) * a.w_stride;
+  const TX* X = reinterpret_cast<const TX*>(a.X) + (int64_t)bi * a.x_stride;
+  const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
+  float acc[4][2] = {};
+  for (int k0 = kbeg; k0 < kend; k0 += BK) {
+    {  // W tile: row tid/4, 8 consecutive k
+      const int r = tid >> 2, kk = (tid & 3) * 8;
+      const int m = m0 + r, k = k0 + kk;
+      float f[8];
+      if (m < a.M && k + 8 <= kend) {
+        load8<TW>(W + (int64_t)m * a.K + k, f);
+      } else {
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+          f[i] = (m < a.M && k + i < kend) ? ldf(W + (int64_t)m * a.K + k + i) : 0.f;
+      }
+#pragma unroll
+      for (int i = 0; i < 8; ++i) Ws[kk + i][r] = f[i];
+    }
+    {  // X tile: token tid/8, 4 consecutive k
+      const int n = tid >> 3, kk = (tid & 7) * 4;
+      const int nn = n0 + n, k = k0 + kk;
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+        Xs[kk + i][n] = (nn < a.N && k + i < kend) ? ldf(X + (int64_t)nn * a.K + k + i) : 0.f;
+    }
+    __syncthreads();
+#pragma unroll 8
+    for (int kk = 0; kk < BK; ++kk) {
+      const float4 w = *reinterpret_cast<const float4*>(&Ws[kk][tx * 4]);
+      const float2 x = *reinterpret_cast<const float2*>(&Xs[kk][ty * 2]);
+      acc[0][0] = fmaf(w.x, x.x, acc[0][0]);
+      acc[1][0] = fmaf(w.y, x.x, acc[1][0]);
+      acc[2][0] = fmaf(w.z, x.x, acc[2][0]);
+      acc[3][0] = fmaf(w.w, x.x, acc[3][0]);
+      acc[0][1] = fmaf(w.x, x.y, acc[0][1]);
+      acc[1][1] = fmaf(w.y, x.y, acc[1][1]);
+      acc[2][1] = fmaf(w.z, x.y, acc[2][1]);
+      acc[3][1] = fmaf(w.w, x.y, acc[3][1]);
+    }
+    __syncthreads();
+  }
+  float* out = a.out + (int64_t)blockIdx.z * a.N * a.M;
+#pragma unroll
+  for (int j = 0; j < 2; ++j) {
+    const int n = n0 + ty * 2 + j;
+    if (n >= a.N) continue;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int m = m0 + tx * 4 + i;
+      if (m < a.M) out[(int64_t)n * a.M + m] = acc[i][j];
+    }
+  }
+}
+
+// ---------------------------------------------------------------- mix
+template <typename T>
+__global__ void __launch_bounds__(kMixThreads) mix_kernel(const MixParams p) {
+  extern __shared__ float sm[];            // alpha[kChanGroup][L], r[L]
+  __shared__ float red[32];
+  float* alpha = sm;
+  float* rl = sm + kChanGroup * p.L;
+  const int b = blockIdx.x, X = blockIdx.y, j0 = blockIdx.z * kChanGroup;
+  const int tid = threadIdx.x;
+  const int nj = min(kChanGroup, p.k - j0);
+  const int kL = p.k * p.L;
+  const T* br = reinterpret_cast<const T*>(p.br[X]);
+  for (int i = tid; i < nj * p.L; i += kMixThreads) {
+    const int o = j0 * p.L + i;  // alpha[j][l] = z[j*L + l]
+    float z = ldf(br + o);
+    for (int s = 0; s < p.nsplit_r; ++s)
+      z += p.zpart[(((int64_t)X * p.nsplit_r + s) * p.B + b) * kL + o];
+    alpha[i] = z;
+  }
+  for (int i = tid; i < p.L; i += kMixThreads) rl[i] = p.inv_rms[b * p.L + i];
+  __syncthreads();
+
+  const T* hp = reinterpret_cast<const T*>(p.h) + (int64_t)b * p.L * p.D;
+  const T* g = reinterpret_cast<const T*>(p.pre_g[X]);
+  float acc[kChanGroup][kMaxEPT];
+#pragma unroll
+  for (int jj = 0; jj < kChanGroup; ++jj)
+#pragma unroll
+    for (int i = 0; i < kMaxEPT; ++i) acc[jj][i] = 0.f;
+  for (int l = 0; l < p.L; ++l) {
+    const float r = rl[l];
+#pragma unroll
+    for (int i = 0; i < kMaxEPT; ++i) {
+      const int e = tid + i * kMixThreads;
+      if (e < p.D) {
+        const float hv = ldf(hp + (int64_t)l * p.D + e) * r * ldf(g + e);
+#pragma unroll
+        for (int jj = 0; jj < kChanGroup; ++jj)
+          if (jj < nj) acc[jj][i] = fmaf(alpha[jj * p.L + l], hv, acc[jj][i]);
+      }
+    }
+  }
+  T* xop = reinterpret_cast<T*>(p.xop);
+#pragma unroll
+  for (int jj = 0; jj < kChanGroup; ++jj) {
+    if (jj >= nj) break;
+    float ss = 0.f;
+#pragma unroll
+    for (int i = 0; i < kMaxEPT; ++i) ss = fmaf(acc[jj][i], acc[jj][i], ss);
+    ss = block_sum(ss, red);
+    const float rr = rsqrtf(ss / (float)p.D + p.eps_rms);
+    const int j = j0 + jj;
+    const T* cg = reinterpret_cast<const T*>(p.ch_g[X]) + (int64_t)j * p.D;
+    T* xo = xop + (((int64_t)X * p.k + j) * p.B + b) * p.D;
+#pragma unroll
+    for (int i = 0; i < kMaxEPT; ++i) {
+      const int e = tid + i * kMixThreads;
+      if (e < p.D) xo[e] = Elem<T>::from_f(acc[jj][i] * rr * ldf(cg + e));
+    }
+  }
+}
+
+// ---------------------------------------------------------------- epilogue
+template <typename T, int HD>
+__global__ void __launch_bounds__(128) kv_epilogue_kernel(const MixParams p) {
+  constexpr int EPL = HD / 32;  // elements per lane; pairs (e, e + HD/2) share a lane
+  const int b = blockIdx.x, j = blockIdx.y, X = blockIdx.z;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int s = p.slot[b];
+  if (s < 1 || s >= p.max_pages * p.P) {
+    if (threadIdx.x == 0 && j == 0 && X == 0) report(p.status, WM_ERR_BOUNDS);
+    return;
+  }
+  const int pg = p.page_table[(int64_t)b * p.max_pages + (s >> p.log2P)];
+  if (pg < 0 || pg >= p.num_pages) {
+    if (threadIdx.x == 0 && j == 0 && X == 0) report(p.status, WM_ERR_BOUNDS);
+    return;
+  }
+  const int nout = p.Hkv * HD;
+  const float* src = p.proj + (((int64_t)X * p.k + j) * p.B + b) * nout;
+  T* pool = reinterpret_cast<T*>(X == 0 ? p.k_pool : p.v_pool);
+  const int64_t base = (((int64_t)j * p.num_pages + pg) * p.Hkv) * p.P + (s & (p.P - 1));
+  const T* qg = reinterpret_cast<const T*>(p.qk_g) + (int64_t)j * HD;
+  for (int hh = warp; hh < p.Hkv; hh += 4) {
+    float y[EPL];
+#pragma unroll
+    for (int i = 0; i < EPL; ++i) y[i] = src[hh * HD + lane + 32 * i];
+    if (X == 0) {
+      float ss = 0.f;
+#pragma unroll
+      for (int i = 0; i < EPL; ++i) ss = fmaf(y[i], y[i], ss);
+      ss = warp_sum(ss);
+      const float rr = rsqrtf(ss / (float)HD + p.eps_qk);
+#pragma unroll
+      for (int i = 0; i < EPL; ++i) y[i] = y[i] * rr * ldf(qg + lane + 32 * i);
+      // rotate-half RoPE: element e pairs with e + HD/2, both held by this lane
+#pragma unroll
+      for (int i = 0; i < EPL / 2; ++i) {
+        const int e = lane + 32 * i;
+        const float cs = p.rope_cs[((int64_t)b * (HD / 2) + e) * 2];
+        const float sn = p.rope_cs[((int64_t)b * (HD / 2) + e) * 2 + 1];
+        const float x0 = y[i], x1 = y[i + EPL / 2];
+        y[i] = x0 * cs - x1 * sn;
+        y[i + EPL / 2] = x1 * cs + x0 * sn;
+      }
+    }
+    T* dst = pool + (base + (int64_t)hh * p.P) * HD;
+#pragma unroll
+    for (int i = 0; i < EPL; ++i) dst[lane + 32 * i] = Elem<T>::from_f(y[i]);
+  }
+}
+
+template <typename T>
+cudaError_t launch_all(MixParams& p, cudaStream_t s) {
+  const int kL = p.k * p.L;
+  prenorm_kernel<T><<<dim3(p.L, p.B), kMixThreads, 0, s>>>(p);
+  {
+    GemmArgs a{};
+    a.W[0] = p.Wr[0];
+    a.W[1] = p.Wr[1];
+    a.w_stride = 0;
+    a.per_branch = 1;
+    a.X = p.xi;
+    a.x_stride = (int64_t)p.B * p.Lp * p.D;
+    a.out = p.zpart;
+    a.M = kL;
+    a.N = p.B;
+    a.K = p.Lp * p.D;
+    a.nsplit = p.nsplit_r;
+    a.k_per_split = ((a.K + p.nsplit_r - 1) / p.nsplit_r + BK - 1) / BK * BK;
+    dim3 grid((a.M + BM - 1) / BM, (a.N + BN - 1) / BN, 2 * a.nsplit);
+    gemm_wxT_simt<T, float><<<grid, 256, 0, s>>>(a);
+  }
+  {
+    const size_t smem = sizeof(float) * (kChanGroup * p.L + p.L);
+    dim3 grid(p.B, 2, (p.k + kChanGroup - 1) / kChanGroup);
+    mix_kernel<T><<<grid, kMixThreads, smem, s>>>(p);
+  }
+  {
+    GemmArgs a{};
+    a.W[0] = p.Wkv[0];
+    a.W[1] = p.Wkv[1];
+    a.w_stride = (int64_t)p.Hkv * p.d * p.D;
+    a.per_branch = p.k;
+    a.X = p.xop;
+    a.x_stride = (int64_t)p.B * p.D;
+    a.out = p.proj;
+    a.M = p.Hkv * p.d;
+    a.N = p.B;
+    a.K = p.D;
+    a.nsplit = 1;
+    a.k_per_split = p.D;
+    dim3 grid((a.M + BM - 1) / BM, (a.N + BN - 1) / BN, 2 * p.k);
+    gemm_wxT_simt<T, T><<<grid, 256, 0, s>>>(a);
+  }
+  {
+    dim3 grid(p.B, p.k, 2);
+    if (p.d == 64)
+      kv_epilogue_kernel<T, 64><<<grid, 128, 0, s>>>(p);
+    else
+      kv_epilogue_kernel<T, 128><<<grid, 128, 0, s>>>(p);
+  }
+  return cudaGetLastError();
+}
+
+size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+}  // namespace
+
+MixWorkspace mix_workspace_layout(const wm_config& cfg, int32_t B, int sm_count) {
+  MixWorkspace w{};
+  const int Lp = (cfg.L + cfg.p - 1) / cfg.p;
+  const int kL = cfg.k * cfg.L;
+  const int64_t Kr = (int64_t)Lp * cfg.D;
+  const int tiles = 2 * ((kL + BM - 1) / BM) * ((B + BN - 1) / BN);
+  int ns = (2 * sm_count + tiles - 1) / tiles;
+  const int max_split = (int)((Kr + 255) / 256);
+  ns = ns < 1 ? 1 : (ns > max_split ? max_split : ns);
+  // same rounding as the launch: whole BK blocks per split
+  const int64_t kps = ((Kr + ns - 1) / ns + BK - 1) / BK * BK;
+  ns = (int)((Kr + kps - 1) / kps);
+  w.nsplit_r = ns;
+  const size_t esz = cfg.dtype == WM_DT_F32 ? 4 : 2;
+  size_t off = 0;
+  w.inv_rms = off; off += align256(sizeof(float) * B * cfg.L);
+  w.xi = off;      off += align256(sizeof(float) * 2 * (size_t)B * Kr);
+  w.zpart = off;   off += align256(sizeof(float) * 2 * (size_t)ns * B * kL);
+  w.rope_cs = off; off += align256(sizeof(float) * (size_t)B * cfg.d);
+  w.xop = off;     off += align256(esz * 2 * (size_t)cfg.k * B * cfg.D);
+  w.proj = off;    off += align256(sizeof(float) * 2 * (size_t)cfg.k * B * cfg.Hkv * cfg.d);
+  w.total = off;
+  return w;
+}
+
+cudaError_t launch_kv_mix(MixParams& p, int dtype, cudaStream_t s) {
+  if (dtype == WM_DT_F32) return launch_all<float>(p, s);
+  return launch_all<__nv_bfloat16>(p, s);
+}
+
+}  // namespace wm

@@ -1,0 +1,257 @@
+// C ABI of libwm (declared in include/wm.h): argument checks, workspace
+// planning and kernel dispatch.  All device memory belongs to the caller.
+#include <math.h>
+#include <string.h>
+
+#include "internal.h"
+#include "wm.h"
+
+namespace {
+
+constexpr int kMaxDevices = 64;
+int g_sm_count[kMaxDevices];  // per-device attribute cache (0 = not yet read)
+
+int sm_count() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0) return 148;
+  if (dev < kMaxDevices && g_sm_count[dev] > 0) return g_sm_count[dev];
+  int n = 0;
+  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
+    n = 148;
+  if (dev < kMaxDevices) g_sm_count[dev] = n;
+  return n;
+}
+
+bool is_pow2(int x) { return x > 0 && (x & (x - 1)) == 0; }
+int ilog2(int x) {
+  int r = 0;
+  while ((1 << r) < x) ++r;
+  return r;
+}
+size_t elem_size(int dtype) { return dtype == WM_DT_F32 ? 4 : 2; }
+size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
+bool aligned(const void* p, size_t a) { return ((uintptr_t)p % a) == 0; }
+
+// Split of one attention launch into chunks of whole pipeline stages.
+struct AttnPlan {
+  int chunk_slots, max_chunks;
+  size_t off_part_o, off_part_ml, off_counters, total;
+};
+
+AttnPlan attn_plan(const wm_config& c, int32_t B, int32_t max_pages) {
+  AttnPlan pl{};
+  const int stage = wm::attn_stage_slots(c.dtype, c.d);
+  const int64_t max_slots = (int64_t)max_pages * c.page_size;
+  const int64_t stages_total = (max_slots + stage - 1) / stage;
+  const int64_t units = (int64_t)B * c.Hkv;
+  // aim for ~16 waves of 3 resident CTAs per SM when every sequence is full
+  const int64_t target = (int64_t)sm_count() * 3 * 16;
+  int64_t per_unit = (target + units - 1) / units;
+  if (per_unit < 1) per_unit = 1;
+  int64_t chunk_stages = (stages_total + per_unit - 1) / per_unit;
+  const int64_t min_stages = 8;
+  if (chunk_stages < min_stages) chunk_stages = min_stages;
+  pl.chunk_slots = (int)(chunk_stages * stage);
+  pl.max_chunks = (int)((max_slots + pl.chunk_slots - 1) / pl.chunk_slots);
+  const size_t rows = (size_t)B * c.Hq;
+  size_t off = 0;
+  pl.off_part_o = off;
+  off += align256(sizeof(float) * rows * pl.max_chunks * c.d);
+  pl.off_part_ml = off;
+  off += align256(sizeof(float) * rows * pl.max_chunks * 2);
+  pl.off_counters = off;
+  off += align256(sizeof(int32_t) * (size_t)B * c.Hkv);
+  pl.total = off;
+  return pl;
+}
+
+wm_status check_cache(const wm_config& c, const wm_cache* cache) {
+  if (!cache || !cache->k_pool || !cache->v_pool || cache->num_pages < 1) return WM_ERR_INVALID_ARG;
+  if (cache->k != c.k || cache->Hkv != c.Hkv || cache->page_size != c.page_size ||
+      cache->d != c.d || cache->dtype != c.dtype)
+    return WM_ERR_INVALID_ARG;
+  if (!aligned(cache->k_pool, 16) || !aligned(cache->v_pool, 16)) return WM_ERR_INVALID_ARG;
+  return WM_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* wm_status_string(wm_status s) {
+  switch (s) {
+    case WM_OK: return "ok";
+    case WM_ERR_INVALID_ARG: return "invalid argument";
+    case WM_ERR_UNSUPPORTED: return "unsupported configuration";
+    case WM_ERR_CUDA: return "CUDA error";
+    case WM_ERR_BOUNDS: return "index out of bounds (device)";
+    case WM_ERR_TIMEOUT: return "pipeline wait timed out (device)";
+  }
+  return "unknown status";
+}
+
+wm_status wm_config_check(const wm_config* c) {
+  if (!c) return WM_ERR_INVALID_ARG;
+  if (c->L < 1 || c->L > WM_MAX_L || c->k < 1 || c->k > c->L || c->D < 1 || c->Hkv < 1 ||
+      c->Hq < 1 || c->Hq % c->Hkv != 0 || c->d < 2 || c->p < 1 || c->page_size < 1 ||
+      !(c->eps_rms >= 0.f) || !(c->eps_qk >= 0.f) || !(c->rope_theta > 0.0))
+    return WM_ERR_INVALID_ARG;
+  if (c->dtype != WM_DT_F32 && c->dtype != WM_DT_BF16) return WM_ERR_INVALID_ARG;
+  for (int l = 0; l < c->L; ++l)
+    if (c->chan_of_layer[l] < 0 || c->chan_of_layer[l] >= c->k) return WM_ERR_INVALID_ARG;
+  // shapes this library builds
+  if (c->d != 64 && c->d != 128) return WM_ERR_UNSUPPORTED;
+  const int G = c->Hq / c->Hkv;
+  if (G != 1 && G != 2 && G != 4 && G != 8) return WM_ERR_UNSUPPORTED;
+  if (c->D % 8 != 0 || c->D > 4096) return WM_ERR_UNSUPPORTED;
+  if (!is_pow2(c->page_size) || c->page_size > 4096) return WM_ERR_UNSUPPORTED;
+  return WM_OK;
+}
+
+size_t wm_cache_bytes(const wm_config* c, int32_t num_pages) {
+  if (wm_config_check(c) != WM_OK || num_pages < 1) return 0;
+  const size_t pool = (size_t)c->k * num_pages * c->Hkv * c->page_size * c->d * elem_size(c->dtype);
+  return 2 * align256(pool);
+}
+
+wm_status wm_cache_alloc(const wm_config* c, void* dev_buf, size_t bytes, int32_t num_pages,
+                         wm_cache* out) {
+  wm_status st = wm_config_check(c);
+  if (st != WM_OK) return st;
+  if (!dev_buf || !out || num_pages < 1 || !aligned(dev_buf, 256)) return WM_ERR_INVALID_ARG;
+  const size_t need = wm_cache_bytes(c, num_pages);
+  if (need == 0 || bytes < need) return WM_ERR_INVALID_ARG;
+  memset(out, 0, sizeof *out);
+  out->k_pool = dev_buf;
+  out->v_pool = (char*)dev_buf + need / 2;
+  out->num_pages = num_pages;
+  out->k = c->k;
+  out->Hkv = c->Hkv;
+  out->page_size = c->page_size;
+  out->d = c->d;
+  out->dtype = c->dtype;
+  return WM_OK;
+}
+
+size_t wm_decode_attn_workspace(const wm_config* c, int32_t B, int32_t max_pages) {
+  if (wm_config_check(c) != WM_OK || B < 0 || max_pages < 1) return 0;
+  if (B == 0) return 256;
+  return attn_plan(*c, B, max_pages).total;
+}
+
+wm_status wm_decode_attn(const wm_config* c, const wm_cache* cache, int32_t layer, const void* q,
+                         const int32_t* page_table, const int32_t* seq_lens, int32_t B,
+                         int32_t max_pages, void* out, void* workspace, size_t ws_bytes,
+                         int32_t* dev_status, void* stream) {
+  wm_status st = wm_config_check(c);
+  if (st != WM_OK) return st;
+  if ((st = check_cache(*c, cache)) != WM_OK) return st;
+  if (layer < 0 || layer >= c->L || B < 0 || max_pages < 1) return WM_ERR_INVALID_ARG;
+  if ((int64_t)max_pages * c->page_size > INT32_MAX / 2) return WM_ERR_INVALID_ARG;
+  if (B == 0) return WM_OK;
+  if (B > 65535 || c->Hkv > 65535) return WM_ERR_UNSUPPORTED;
+  if (!q || !page_table || !seq_lens || !out || !workspace) return WM_ERR_INVALID_ARG;
+  if (!aligned(q, 16) || !aligned(out, 16) || !aligned(workspace, 256)) return WM_ERR_INVALID_ARG;
+  const AttnPlan pl = attn_plan(*c, B, max_pages);
+  if (ws_bytes < pl.total) return WM_ERR_INVALID_ARG;
+
+  const int chan = c->chan_of_layer[layer];
+  const size_t esz = elem_size(c->dtype);
+  const int64_t chan_elems = (int64_t)cache->num_pages * c->Hkv * c->page_size * c->d;
+  wm::AttnParams p{};
+  p.k_pool = (const char*)cache->k_pool + (size_t)chan * chan_elems * esz;
+  p.v_pool = (const char*)cache->v_pool + (size_t)chan * chan_elems * esz;
+  p.q = q;
+  p.out = out;
+  p.page_table = page_table;
+  p.seq_lens = seq_lens;
+  p.part_o = (float*)((char*)workspace + pl.off_part_o);
+  p.part_ml = (float*)((char*)workspace + pl.off_part_ml);
+  p.counters = (int32_t*)((char*)workspace + pl.off_counters);
+  p.status = dev_status;
+  p.page_stride = (int64_t)c->Hkv * c->page_size * c->d;
+  p.Hq = c->Hq;
+  p.Hkv = c->Hkv;
+  p.P = c->page_size;
+  p.log2P = ilog2(c->page_size);
+  p.num_pages = cache->num_pages;
+  p.max_pages = max_pages;
+  p.chunk_slots = pl.chunk_slots;
+  p.max_chunks = pl.max_chunks;
+  p.qscale = (float)(1.4426950408889634 / sqrt((double)c->d));
+  cudaError_t e = wm::launch_decode_attn(p, c->dtype, c->d, c->Hq / c->Hkv, B, c->Hkv,
+                                         (cudaStream_t)stream);
+  return e == cudaSuccess ? WM_OK : WM_ERR_CUDA;
+}
+
+size_t wm_kv_mix_workspace(const wm_config* c, int32_t B) {
+  if (wm_config_check(c) != WM_OK || B < 0) return 0;
+  if (B == 0) return 256;
+  return wm::mix_workspace_layout(*c, B, sm_count()).total;
+}
+
+wm_status wm_kv_mix(const wm_config* c, const wm_cache* cache, const wm_mix_weights* w,
+                    const void* h, const int32_t* page_table, const int32_t* slot, int32_t B,
+                    int32_t max_pages, void* workspace, size_t ws_bytes, int32_t* dev_status,
+                    void* stream) {
+  wm_status st = wm_config_check(c);
+  if (st != WM_OK) return st;
+  if ((st = check_cache(*c, cache)) != WM_OK) return st;
+  if (B < 0 || max_pages < 1 || !w) return WM_ERR_INVALID_ARG;
+  if ((int64_t)max_pages * c->page_size > INT32_MAX / 2) return WM_ERR_INVALID_ARG;
+  if (B == 0) return WM_OK;
+  if (B > 65535) return WM_ERR_UNSUPPORTED;
+  if (!h || !page_table || !slot || !workspace || !w->qk_g) return WM_ERR_INVALID_ARG;
+  for (int X = 0; X < 2; ++X)
+    if (!w->pre_g[X] || !w->Wr[X] || !w->br[X] || !w->ch_g[X] || !w->Wkv[X])
+      return WM_ERR_INVALID_ARG;
+  for (int X = 0; X < 2; ++X)
+    if (!aligned(w->Wr[X], 16) || !aligned(w->Wkv[X], 16)) return WM_ERR_INVALID_ARG;
+  if (!aligned(workspace, 256)) return WM_ERR_INVALID_ARG;
+  const wm::MixWorkspace ws = wm::mix_workspace_layout(*c, B, sm_count());
+  if (ws_bytes < ws.total) return WM_ERR_INVALID_ARG;
+
+  wm::MixParams p{};
+  p.B = B;
+  p.L = c->L;
+  p.k = c->k;
+  p.D = c->D;
+  p.Hkv = c->Hkv;
+  p.d = c->d;
+  p.p = c->p;
+  p.Lp = (c->L + c->p - 1) / c->p;
+  p.P = c->page_size;
+  p.log2P = ilog2(c->page_size);
+  p.num_pages = cache->num_pages;
+  p.max_pages = max_pages;
+  p.eps_rms = c->eps_rms;
+  p.eps_qk = c->eps_qk;
+  p.h = h;
+  for (int X = 0; X < 2; ++X) {
+    p.pre_g[X] = w->pre_g[X];
+    p.Wr[X] = w->Wr[X];
+    p.br[X] = w->br[X];
+    p.ch_g[X] = w->ch_g[X];
+    p.Wkv[X] = w->Wkv[X];
+  }
+  p.qk_g = w->qk_g;
+  p.page_table = page_table;
+  p.slot = slot;
+  p.k_pool = cache->k_pool;
+  p.v_pool = cache->v_pool;
+  char* base = (char*)workspace;
+  p.inv_rms = (float*)(base + ws.inv_rms);
+  p.xi = (float*)(base + ws.xi);
+  p.zpart = (float*)(base + ws.zpart);
+  p.rope_cs = (float*)(base + ws.rope_cs);
+  p.xop = base + ws.xop;
+  p.proj = (float*)(base + ws.proj);
+  p.nsplit_r = ws.nsplit_r;
+  p.status = dev_status;
+  for (int i = 0; i < c->d / 2 && i < wm::kMaxRopeHalf; ++i)
+    p.inv_freq[i] = pow(c->rope_theta, -2.0 * i / c->d);
+  cudaError_t e = wm::launch_kv_mix(p, c->dtype, (cudaStream_t)stream);
+  return e == cudaSuccess ? WM_OK : WM_ERR_CUDA;
+}
+
+}  // extern "C"

@@ -1,0 +1,99 @@
+"""The C-ABI library loads, exports every entry point include/*.h declares,
+and rejects bad arguments on the host (no GPU needed, nothing launched)."""
+import ctypes
+import glob
+import os
+import re
+
+import pytest
+
+from paper_2608_18486_gb300 import _lib as W
+from wm_synth import configs
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def declared_functions():
+    names = set()
+    for hdr in glob.glob(os.path.join(ROOT, "include", "*.h")):
+        text = re.sub(r"/\*.*?\*/", "", open(hdr).read(), flags=re.S)
+        names |= set(re.findall(r"\b(wm_\w+)\s*\(", text))
+    return sorted(names)
+
+
+def test_library_exports_every_declared_entry_point():
+    lib = ctypes.CDLL(W.LIB_PATH)
+    names = declared_functions()
+    assert set(W.EXPORTED) <= set(names)
+    missing = [n for n in names if not hasattr(lib, n)]
+    assert not missing, missing
+
+
+def cfg(**kw):
+    w = configs.get("large")
+    c = W.make_config(w.L, w.k, w.D, w.Hq, w.Hkv, w.d, w.p, w.page, w.dtype, w.chan_of_layer())
+    for k, v in kw.items():
+        setattr(c, k, v)
+    return c
+
+
+@pytest.mark.parametrize("field,value,code", [
+    ("k", 33, W.WM_ERR_INVALID_ARG), ("k", 0, W.WM_ERR_INVALID_ARG),
+    ("Hq", 33, W.WM_ERR_INVALID_ARG), ("p", 0, W.WM_ERR_INVALID_ARG),
+    ("dtype", 7, W.WM_ERR_INVALID_ARG), ("d", 96, W.WM_ERR_UNSUPPORTED),
+    ("page_size", 24, W.WM_ERR_UNSUPPORTED), ("D", 8192, W.WM_ERR_UNSUPPORTED),
+    ("Hq", 96, W.WM_ERR_UNSUPPORTED)])
+def test_config_check_codes(field, value, code):
+    assert W.wm_config_check(cfg()) == W.WM_OK
+    assert W.wm_config_check(cfg(**{field: value})) == code
+
+
+def test_channel_map_must_point_at_existing_channels():
+    c = cfg()
+    c.chan_of_layer[5] = c.k
+    assert W.wm_config_check(c) == W.WM_ERR_INVALID_ARG
+
+
+def test_cache_sizing_and_layout_without_gpu():
+    c = cfg()
+    n = W.wm_cache_bytes(c, 10)
+    pool = c.k * 10 * c.Hkv * c.page_size * c.d * 2
+    assert n == 2 * ((pool + 255) // 256 * 256)
+    fake = 1 << 40  # never dereferenced: wm_cache_alloc only lays out views
+    cache = W.wm_cache_alloc(c, fake, n, 10)
+    assert cache.k_pool == fake and cache.v_pool == fake + n // 2
+    with pytest.raises(W.WMError):
+        W.wm_cache_alloc(c, fake, n - 1, 10)
+    with pytest.raises(W.WMError):
+        W.wm_cache_alloc(c, fake + 8, n, 10)
+    assert W.wm_cache_bytes(c, 0) == 0
+
+
+def test_compute_calls_reject_bad_arguments_before_launching():
+    c = cfg()
+    n = W.wm_cache_bytes(c, 4)
+    cache = W.wm_cache_alloc(c, 1 << 40, n, 4)
+    fake = 1 << 41
+    ws = W.wm_decode_attn_workspace(c, 2, 4)
+    assert ws > 0
+    # layer out of range, NULL query, misaligned output, short workspace
+    assert W.wm_decode_attn(c, cache, c.L, fake, fake, fake, 2, 4, fake, fake, ws, None, None) == W.WM_ERR_INVALID_ARG
+    assert W.wm_decode_attn(c, cache, 0, None, fake, fake, 2, 4, fake, fake, ws, None, None) == W.WM_ERR_INVALID_ARG
+    assert W.wm_decode_attn(c, cache, 0, fake, fake, fake, 2, 4, fake + 2, fake, ws, None, None) == W.WM_ERR_INVALID_ARG
+    assert W.wm_decode_attn(c, cache, 0, fake, fake, fake, 2, 4, fake, fake, ws - 1, None, None) == W.WM_ERR_INVALID_ARG
+    # empty batch is a no-op even with NULL buffers
+    assert W.wm_decode_attn(c, cache, 0, None, None, None, 0, 4, None, None, 0, None, None) == W.WM_OK
+    # a cache laid out for another config is refused
+    other = cfg(k=8)
+    assert W.wm_decode_attn(other, cache, 0, fake, fake, fake, 2, 4, fake, fake, ws, None, None) == W.WM_ERR_INVALID_ARG
+    wts = W.mix_weights((fake, fake), (fake, fake), (fake, fake), (fake, fake), (fake, fake), fake)
+    mws = W.wm_kv_mix_workspace(c, 2)
+    assert W.wm_kv_mix(c, cache, wts, fake, fake, fake, 2, 4, fake, mws - 1, None, None) == W.WM_ERR_INVALID_ARG
+    bad = W.mix_weights((fake, fake), (fake, None), (fake, fake), (fake, fake), (fake, fake), fake)
+    assert W.wm_kv_mix(c, cache, bad, fake, fake, fake, 2, 4, fake, mws, None, None) == W.WM_ERR_INVALID_ARG
+    assert W.wm_kv_mix(c, cache, wts, None, None, None, 0, 4, None, 0, None, None) == W.WM_OK
+
+
+def test_status_strings():
+    for code in range(6):
+        assert W.wm_status_string(code) and W.wm_status_string(code) != "unknown status"

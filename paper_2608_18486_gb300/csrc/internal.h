@@ -16,17 +16,20 @@ struct AttnParams {
   void* out;              // [B][Hq][d]
   const int32_t* page_table;
   const int32_t* seq_lens;
-  float* part_o;          // [B*Hq][max_chunks][d]
-  float* part_ml;         // [B*Hq][max_chunks][2] (max, sum) in log2 units
+  float* part_o;          // [2][nwarps][G][d]: first / last piece partial of each warp
+  float* part_ml;         // [2][nwarps][G][2]: (max, sum) in log2 units
   int32_t* counters;      // [B*Hkv] arrival tickets, zero between launches
   int32_t* status;
   int64_t page_stride;    // elements between consecutive physical pages
-  int32_t Hq, Hkv, P, log2P, num_pages, max_pages, chunk_slots, max_chunks;
+  int32_t B, Hq, Hkv, P, log2P, num_pages, max_pages;
+  int32_t nwarps;         // warps of the launch grid
   float qscale;           // log2(e) / sqrt(d)
 };
 
 int attn_stage_slots(int dtype, int d);
-cudaError_t launch_decode_attn(const AttnParams& p, int dtype, int d, int G, int B, int Hkv,
+int attn_warps_per_cta();
+size_t attn_smem_bytes(int dtype, int d, int G, int B);
+cudaError_t launch_decode_attn(const AttnParams& p, int dtype, int d, int G, int grid,
                                cudaStream_t s);
 
 // ------------------------------------------------------------ KV pool (mix)
@@ -68,5 +71,9 @@ struct MixWorkspace {
 
 MixWorkspace mix_workspace_layout(const wm_config& cfg, int32_t B, int sm_count);
 cudaError_t launch_kv_mix(MixParams& p, int dtype, cudaStream_t s);
+
+// tcgen05 projection with the fused key/value epilogue (bf16 only)
+bool proj_tc_supported(const MixParams& p);
+cudaError_t launch_proj_tc(const MixParams& p, cudaStream_t s);
 
 }  // namespace wm

@@ -300,6 +300,12 @@ cudaError_t launch_all(MixParams& p, cudaStream_t s) {
     dim3 grid(p.B, 2, (p.k + kChanGroup - 1) / kChanGroup);
     mix_kernel<T><<<grid, kMixThreads, smem, s>>>(p);
   }
+  if (sizeof(T) == 2 && proj_tc_supported(p)) {
+    // bf16: tensor-core projection, QK-norm, RoPE and cache write in one kernel
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    return launch_proj_tc(p, s);
+  }
   {
     GemmArgs a{};
     a.W[0] = p.Wkv[0];

@@ -32,33 +32,34 @@ size_t elem_size(int dtype) { return dtype == WM_DT_F32 ? 4 : 2; }
 size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 bool aligned(const void* p, size_t a) { return ((uintptr_t)p % a) == 0; }
 
-// Split of one attention launch into chunks of whole pipeline stages.
+// Persistent grid of one attention launch and its workspace layout.
 struct AttnPlan {
-  int chunk_slots, max_chunks;
+  int grid, nwarps;
   size_t off_part_o, off_part_ml, off_counters, total;
 };
+
+constexpr int kAttnCtasPerSm = 2;
+constexpr int kAttnMaxBatch = 4096;
 
 AttnPlan attn_plan(const wm_config& c, int32_t B, int32_t max_pages) {
   AttnPlan pl{};
   const int stage = wm::attn_stage_slots(c.dtype, c.d);
   const int64_t max_slots = (int64_t)max_pages * c.page_size;
-  const int64_t stages_total = (max_slots + stage - 1) / stage;
-  const int64_t units = (int64_t)B * c.Hkv;
-  // aim for ~16 waves of 3 resident CTAs per SM when every sequence is full
-  const int64_t target = (int64_t)sm_count() * 3 * 16;
-  int64_t per_unit = (target + units - 1) / units;
-  if (per_unit < 1) per_unit = 1;
-  int64_t chunk_stages = (stages_total + per_unit - 1) / per_unit;
-  const int64_t min_stages = 8;
-  if (chunk_stages < min_stages) chunk_stages = min_stages;
-  pl.chunk_slots = (int)(chunk_stages * stage);
-  pl.max_chunks = (int)((max_slots + pl.chunk_slots - 1) / pl.chunk_slots);
-  const size_t rows = (size_t)B * c.Hq;
+  const int64_t ns_max = (int64_t)B * c.Hkv * ((max_slots + stage - 1) / stage);
+  const int wpc = wm::attn_warps_per_cta();
+  // one CTA pair per SM, fewer when there are under 4 stages per warp
+  int64_t grid = (int64_t)sm_count() * kAttnCtasPerSm;
+  const int64_t by_work = (ns_max + 4 * wpc - 1) / (4 * wpc);
+  if (by_work < grid) grid = by_work;
+  if (grid < 1) grid = 1;
+  pl.grid = (int)grid;
+  pl.nwarps = (int)grid * wpc;
+  const int G = c.Hq / c.Hkv;
   size_t off = 0;
   pl.off_part_o = off;
-  off += align256(sizeof(float) * rows * pl.max_chunks * c.d);
+  off += align256(sizeof(float) * 2 * (size_t)pl.nwarps * G * c.d);
   pl.off_part_ml = off;
-  off += align256(sizeof(float) * rows * pl.max_chunks * 2);
+  off += align256(sizeof(float) * 2 * (size_t)pl.nwarps * G * 2);
   pl.off_counters = off;
   off += align256(sizeof(int32_t) * (size_t)B * c.Hkv);
   pl.total = off;
@@ -149,7 +150,7 @@ wm_status wm_decode_attn(const wm_config* c, const wm_cache* cache, int32_t laye
   if (layer < 0 || layer >= c->L || B < 0 || max_pages < 1) return WM_ERR_INVALID_ARG;
   if ((int64_t)max_pages * c->page_size > INT32_MAX / 2) return WM_ERR_INVALID_ARG;
   if (B == 0) return WM_OK;
-  if (B > 65535 || c->Hkv > 65535) return WM_ERR_UNSUPPORTED;
+  if (B > kAttnMaxBatch) return WM_ERR_UNSUPPORTED;
   if (!q || !page_table || !seq_lens || !out || !workspace) return WM_ERR_INVALID_ARG;
   if (!aligned(q, 16) || !aligned(out, 16) || !aligned(workspace, 256)) return WM_ERR_INVALID_ARG;
   const AttnPlan pl = attn_plan(*c, B, max_pages);
@@ -176,10 +177,10 @@ wm_status wm_decode_attn(const wm_config* c, const wm_cache* cache, int32_t laye
   p.log2P = ilog2(c->page_size);
   p.num_pages = cache->num_pages;
   p.max_pages = max_pages;
-  p.chunk_slots = pl.chunk_slots;
-  p.max_chunks = pl.max_chunks;
+  p.B = B;
+  p.nwarps = pl.nwarps;
   p.qscale = (float)(1.4426950408889634 / sqrt((double)c->d));
-  cudaError_t e = wm::launch_decode_attn(p, c->dtype, c->d, c->Hq / c->Hkv, B, c->Hkv,
+  cudaError_t e = wm::launch_decode_attn(p, c->dtype, c->d, c->Hq / c->Hkv, pl.grid,
                                          (cudaStream_t)stream);
   return e == cudaSuccess ? WM_OK : WM_ERR_CUDA;
 }

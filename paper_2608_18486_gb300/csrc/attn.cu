@@ -33,19 +33,36 @@ namespace {
 constexpr int kWarps = 4;
 constexpr int kThreads = kWarps * 32;
 constexpr int kWStages = 3;          // ring depth per warp
-constexpr int kWStageBytes = 8192;   // K + V bytes per stage
 
-template <typename T, int HD>
+// SB: K + V bytes of one pipeline stage (4 KB or 8 KB).
+template <typename T, int HD, int SB>
 struct Shape {
-  static constexpr int VEC = Elem<T>::kVec;                       // elements per lane load
-  static constexpr int LPS = HD / VEC;                            // lanes per slot
+  // A quarter warp (8 lanes) covers each 128-byte run of a slot row, so every
+  // 16-byte shared load of the warp is bank-conflict free.
+  static constexpr int VEC = Elem<T>::kVec;                       // elements per 16 bytes
+  static constexpr int LPS = 8;                                   // lanes per slot
   static constexpr int SPW = 32 / LPS;                            // slots per warp step
-  static constexpr int STAGE_SLOTS = kWStageBytes / (2 * HD * (int)sizeof(T));
+  static constexpr int NVL = HD * (int)sizeof(T) / (16 * LPS);    // 16-byte vectors per lane
+  static constexpr int EPL = NVL * VEC;                           // elements per lane
+  static constexpr int STAGE_SLOTS = SB / (2 * HD * (int)sizeof(T));
   static constexpr int STAGE_ELEMS = STAGE_SLOTS * HD;
   static constexpr int ITERS = STAGE_SLOTS / SPW;
-  static_assert(LPS >= 1 && LPS <= 32 && (32 % LPS) == 0, "lane split");
+  static_assert(NVL >= 1 && HD * (int)sizeof(T) == NVL * 16 * LPS, "lane split");
   static_assert(ITERS >= 1 && STAGE_SLOTS % SPW == 0 && STAGE_SLOTS <= 32, "stage split");
 };
+
+// Lane part `lp` owns the 16-byte vectors lp, lp + 8, ... of a slot row.
+template <typename T, int HD, int SB>
+__device__ __forceinline__ void load_row(const T* row, int lp, float2 (&f)[Shape<T, HD, SB>::EPL / 2]) {
+  using SH = Shape<T, HD, SB>;
+#pragma unroll
+  for (int v = 0; v < SH::NVL; ++v) {
+    float t[SH::VEC];
+    Elem<T>::unpack(*reinterpret_cast<const uint4*>(row + (v * SH::LPS + lp) * SH::VEC), t);
+#pragma unroll
+    for (int i = 0; i < SH::VEC / 2; ++i) f[v * SH::VEC / 2 + i] = make_float2(t[2 * i], t[2 * i + 1]);
+  }
+}
 
 template <typename T>
 __device__ __forceinline__ void store_vec(T* dst, const float* v);
@@ -98,13 +115,101 @@ __device__ __forceinline__ int64_t warp_of(int64_t x, int64_t NS, int64_t GW) {
   return ((x + 1) * GW - 1) / NS;
 }
 
-template <typename T, int HD, int G>
-__global__ void __launch_bounds__(kThreads) decode_attn_kernel(const AttnParams p) {
-  using SH = Shape<T, HD>;
-  constexpr int VEC = SH::VEC, LPS = SH::LPS, SPW = SH::SPW;
-  constexpr int STAGE_SLOTS = SH::STAGE_SLOTS, STAGE_ELEMS = SH::STAGE_ELEMS, ITERS = SH::ITERS;
+// Online-softmax state of one lane: G query heads, EPL output elements each.
+template <typename T, int HD, int G, int SB>
+struct SoftState {
+  float m[G], l[G];
+  float2 acc[G][Shape<T, HD, SB>::EPL / 2];
+};
+
+// One pipeline stage of K/V rows for this warp's current piece.  FULL: every
+// slot of the stage is inside the sequence and on a fetched page, so no
+// masking is needed; otherwise masked slots never touch the sums (NaN-safe).
+template <typename T, int HD, int G, int SB, bool FULL>
+__device__ __forceinline__ void consume_stage(const T* Ks, const T* Vs, int lane_slot, int lane_part,
+                                              const float2 (&q2)[G][Shape<T, HD, SB>::EPL / 2],
+                                              float qscale, int valid_slots, uint64_t mask,
+                                              int log2P_in_stage, SoftState<T, HD, G, SB>& st) {
+  using SH = Shape<T, HD, SB>;
+  constexpr int SPW = SH::SPW, ITERS = SH::ITERS, E2 = SH::EPL / 2;
+  float sc[G][ITERS];
+#pragma unroll
+  for (int it = 0; it < ITERS; ++it) {
+    const int ls = it * SPW + lane_slot;
+    float2 kf[E2];
+    load_row<T, HD, SB>(Ks + ls * HD, lane_part, kf);
+    bool valid = true;
+    if (!FULL) valid = (ls < valid_slots) && ((mask >> (ls >> log2P_in_stage)) & 1ull);
+#pragma unroll
+    for (int g = 0; g < G; ++g) {
+      float2 a = make_float2(0.f, 0.f);
+#pragma unroll
+      for (int i = 0; i < E2; ++i) a = __ffma2_rn(q2[g][i], kf[i], a);
+      float s = group_sum<SH::LPS>(a.x + a.y) * qscale;
+      sc[g][it] = valid ? s : -INFINITY;
+    }
+  }
+#pragma unroll
+  for (int g = 0; g < G; ++g) {
+    float mx = sc[g][0];
+#pragma unroll
+    for (int it = 1; it < ITERS; ++it) mx = fmaxf(mx, sc[g][it]);
+    const float mnew = fmaxf(st.m[g], mx);
+    if (FULL || mnew != -INFINITY) {
+      const float corr = exp2f(st.m[g] - mnew);  // 0 while m is still -inf
+      st.l[g] *= corr;
+      const float2 c2 = make_float2(corr, corr);
+#pragma unroll
+      for (int i = 0; i < E2; ++i) st.acc[g][i] = __fmul2_rn(st.acc[g][i], c2);
+      st.m[g] = mnew;
+    }
+  }
+#pragma unroll
+  for (int it = 0; it < ITERS; ++it) {
+    const int ls = it * SPW + lane_slot;
+    float2 vf[E2];
+    load_row<T, HD, SB>(Vs + ls * HD, lane_part, vf);
+#pragma unroll
+    for (int g = 0; g < G; ++g) {
+      if (FULL || sc[g][it] != -INFINITY) {
+        const float pr = exp2f(sc[g][it] - st.m[g]);
+        st.l[g] += pr;
+        const float2 p2 = make_float2(pr, pr);
+#pragma unroll
+        for (int i = 0; i < E2; ++i) st.acc[g][i] = __ffma2_rn(p2, vf[i], st.acc[g][i]);
+      }
+    }
+  }
+}
+
+// Write G rows of d outputs (lanes of slot group 0 own vectors lane, lane+8, ...).
+template <typename T, int HD, int G, int SB>
+__device__ __forceinline__ void write_rows(T* out_rows, int lane_part, const SoftState<T, HD, G, SB>& st) {
+  using SH = Shape<T, HD, SB>;
+#pragma unroll
+  for (int g = 0; g < G; ++g) {
+    const float inv = st.l[g] > 0.f ? 1.f / st.l[g] : 0.f;
+#pragma unroll
+    for (int v = 0; v < SH::NVL; ++v) {
+      float o[SH::VEC];
+#pragma unroll
+      for (int i = 0; i < SH::VEC / 2; ++i) {
+        o[2 * i] = st.acc[g][v * SH::VEC / 2 + i].x * inv;
+        o[2 * i + 1] = st.acc[g][v * SH::VEC / 2 + i].y * inv;
+      }
+      store_vec<T>(out_rows + g * HD + (v * SH::LPS + lane_part) * SH::VEC, o);
+    }
+  }
+}
+
+template <typename T, int HD, int G, int SB>
+__global__ void __launch_bounds__(kThreads, SB == 4096 ? 4 : 2) decode_attn_kernel(const AttnParams p) {
+  using SH = Shape<T, HD, SB>;
+  constexpr int VEC = SH::VEC, LPS = SH::LPS, E2 = SH::EPL / 2;
+  constexpr int STAGE_SLOTS = SH::STAGE_SLOTS, STAGE_ELEMS = SH::STAGE_ELEMS;
   constexpr uint32_t KV_BYTES = STAGE_ELEMS * sizeof(T);
   constexpr uint32_t Q_BYTES = G * HD * sizeof(T);
+  constexpr unsigned FULLMASK = 0xFFFFFFFFu;
 
   extern __shared__ __align__(128) unsigned char smem_raw[];
   T* ring = reinterpret_cast<T*>(smem_raw);                       // [W][S][2][STAGE_ELEMS]
@@ -118,6 +223,12 @@ __global__ void __launch_bounds__(kThreads) decode_attn_kernel(const AttnParams 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int B = p.B, Hkv = p.Hkv;
   const int max_slots = p.max_pages * p.P;
+
+  // Programmatic dependent launch: the next grid on the stream may be
+  // scheduled now (it waits for this one before reading anything), and this
+  // grid waits here until the previous one has finished and flushed.
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  asm volatile("griddepcontrol.wait;" ::: "memory");
 
   // ---- stages per sequence and their prefix sums (every CTA, all threads)
   {
@@ -172,6 +283,30 @@ __global__ void __launch_bounds__(kThreads) decode_attn_kernel(const AttnParams 
   const uint64_t policy = l2_evict_first_policy();
   const int lane_slot = lane / LPS, lane_part = lane % LPS;
 
+  // ---- page-table window of the producer: lane i holds the page id of
+  // logical page win0 + i (cur) and win0 + 32 + i (nxt) of sequence win_b.
+  int win_b = -1, win0 = 0, pg_cur = -1, pg_nxt = -1;
+  auto load_pg = [&](int b, int lp) -> int {
+    return lp < p.max_pages ? __ldg(p.page_table + (int64_t)b * p.max_pages + lp) : -1;
+  };
+  // page id of logical page lp + (this lane's offset) -- all lanes call it together
+  auto page_of = [&](int b, int lp, int lane_off) -> int {
+    if (b != win_b || lp < win0 || lp >= win0 + 64) {
+      win_b = b;
+      win0 = lp;
+      pg_cur = load_pg(b, lp + lane);
+      pg_nxt = load_pg(b, lp + 32 + lane);
+    } else if (lp >= win0 + 32) {
+      win0 += 32;
+      pg_cur = pg_nxt;
+      pg_nxt = load_pg(b, win0 + 32 + lane);
+    }
+    const int idx = lp + lane_off - win0;  // 0 .. 63
+    const int a = __shfl_sync(FULLMASK, pg_cur, idx & 31);
+    const int c = __shfl_sync(FULLMASK, pg_nxt, idx & 31);
+    return idx < 32 ? a : c;
+  };
+
   // ---- producer: stage xp at cursor pc into ring slot buf
   Cursor pc = locate(x0, pre, B, Hkv);
   int64_t xp = x0;
@@ -179,7 +314,6 @@ __global__ void __launch_bounds__(kThreads) decode_attn_kernel(const AttnParams 
     const bool first = (xp == x0) || pc.st == 0;
     const int S = lens[pc.b];
     const int s_begin = pc.st * STAGE_SLOTS;
-    const int32_t* pt = p.page_table + (int64_t)pc.b * p.max_pages;
     const T* kb = reinterpret_cast<const T*>(p.k_pool) + (int64_t)pc.h * p.P * HD;
     const T* vb = reinterpret_cast<const T*>(p.v_pool) + (int64_t)pc.h * p.P * HD;
     T* kd = myring + buf * 2 * STAGE_ELEMS;
@@ -188,8 +322,8 @@ __global__ void __launch_bounds__(kThreads) decode_attn_kernel(const AttnParams 
     const uint32_t qb = first ? Q_BYTES : 0u;
     const T* qsrc = reinterpret_cast<const T*>(p.q) + ((int64_t)pc.b * p.Hq + pc.h * G) * HD;
     if (p.P >= STAGE_SLOTS) {
+      const int pg = page_of(pc.b, s_begin >> p.log2P, 0);
       if (lane == 0) {
-        const int pg = pt[s_begin >> p.log2P];
         const bool ok = pg >= 0 && pg < p.num_pages;
         masks[warp][buf] = ok ? 1ull : 0ull;
         if (!ok) report(p.status, WM_ERR_BOUNDS);
@@ -202,13 +336,12 @@ __global__ void __launch_bounds__(kThreads) decode_attn_kernel(const AttnParams 
         if (first) bulk_g2s(myq + buf * G * HD, qsrc, Q_BYTES, bar, policy);
       }
     } else {
-      const int npp = STAGE_SLOTS >> p.log2P;           // pages per stage (<= 32)
+      const int npp = STAGE_SLOTS >> p.log2P;  // pages per stage (<= 32)
       const int lp0 = s_begin >> p.log2P;
       const int lpn = min(npp, ((S - 1) >> p.log2P) - lp0 + 1);
-      int pg = -1;
-      if (lane < lpn) pg = pt[lp0 + lane];
+      const int pg = page_of(pc.b, lp0, lane < lpn ? lane : 0);
       const bool ok = lane < lpn && pg >= 0 && pg < p.num_pages;
-      const uint32_t mask = __ballot_sync(0xFFFFFFFFu, ok);
+      const uint32_t mask = __ballot_sync(FULLMASK, ok);
       const uint32_t bytes = (uint32_t)p.P * HD * sizeof(T);
       if (lane == 0) {
         masks[warp][buf] = mask;
@@ -230,15 +363,17 @@ __global__ void __launch_bounds__(kThreads) decode_attn_kernel(const AttnParams 
   for (int s = 0; s < kWStages && xp < x1; ++s) issue(s);
 
   // ---- consumer
+  const int log2P_in_stage = p.P >= STAGE_SLOTS ? 30 : p.log2P;  // stage page index = slot >> this
+  const uint64_t all_pages = p.P >= STAGE_SLOTS ? 1ull : ((1ull << (STAGE_SLOTS >> p.log2P)) - 1ull);
   Cursor cc = locate(x0, pre, B, Hkv);
   bool piece_first = true;  // the piece that starts at x0 is this warp's first
-  float qv[G][VEC];
-  float m[G], l[G], acc[G][VEC];
+  float2 q2[G][E2];
+  SoftState<T, HD, G, SB> st;
   for (int64_t x = x0; x < x1; ++x) {
     const int buf = (int)((x - x0) % kWStages);
     const uint32_t parity = (uint32_t)(((x - x0) / kWStages) & 1);
     const bool ok = mbar_wait(&bars[warp][buf], parity);
-    if (__any_sync(0xFFFFFFFFu, !ok)) {
+    if (__any_sync(FULLMASK, !ok)) {
       // a copy never landed: report, drain what is in flight (bounded) and stop
       if (lane == 0) {
         report(p.status, WM_ERR_TIMEOUT);
@@ -248,114 +383,62 @@ __global__ void __launch_bounds__(kThreads) decode_attn_kernel(const AttnParams 
       __syncwarp();
       return;
     }
-    const bool start = (x == x0) || cc.st == 0;
-    if (start) {
-      const T* qs = myq + buf * G * HD + lane_part * VEC;
+    if ((x == x0) || cc.st == 0) {
+      const T* qs = myq + buf * G * HD;
 #pragma unroll
       for (int g = 0; g < G; ++g) {
-        float f[VEC];
-        Elem<T>::unpack(*reinterpret_cast<const uint4*>(qs + g * HD), f);
+        load_row<T, HD, SB>(qs + g * HD, lane_part, q2[g]);
+        st.m[g] = -INFINITY;
+        st.l[g] = 0.f;
 #pragma unroll
-        for (int v = 0; v < VEC; ++v) qv[g][v] = f[v] * p.qscale;
-        m[g] = -INFINITY;
-        l[g] = 0.f;
-#pragma unroll
-        for (int v = 0; v < VEC; ++v) acc[g][v] = 0.f;
+        for (int i = 0; i < E2; ++i) st.acc[g][i] = make_float2(0.f, 0.f);
       }
     }
-    const int S = lens[cc.b];
-    const int s_begin = cc.st * STAGE_SLOTS;
+    const int valid_slots = lens[cc.b] - cc.st * STAGE_SLOTS;
     const uint64_t mask = masks[warp][buf];
     const T* Ks = myring + buf * 2 * STAGE_ELEMS;
     const T* Vs = Ks + STAGE_ELEMS;
-    float sc[G][ITERS];
-#pragma unroll
-    for (int it = 0; it < ITERS; ++it) {
-      const int ls = it * SPW + lane_slot;
-      float kf[VEC];
-      Elem<T>::unpack(*reinterpret_cast<const uint4*>(Ks + ls * HD + lane_part * VEC), kf);
-      const int pidx = (p.P >= STAGE_SLOTS) ? 0 : (ls >> p.log2P);
-      const bool valid = (s_begin + ls < S) && ((mask >> pidx) & 1ull);
-#pragma unroll
-      for (int g = 0; g < G; ++g) {
-        float s = 0.f;
-#pragma unroll
-        for (int v = 0; v < VEC; ++v) s = fmaf(qv[g][v], kf[v], s);
-        s = group_sum<LPS>(s);
-        sc[g][it] = valid ? s : -INFINITY;
-      }
-    }
-#pragma unroll
-    for (int g = 0; g < G; ++g) {
-      float mx = sc[g][0];
-#pragma unroll
-      for (int it = 1; it < ITERS; ++it) mx = fmaxf(mx, sc[g][it]);
-      const float mnew = fmaxf(m[g], mx);
-      if (mnew != -INFINITY) {
-        const float corr = exp2f(m[g] - mnew);  // 0 while m is still -inf
-        l[g] *= corr;
-#pragma unroll
-        for (int v = 0; v < VEC; ++v) acc[g][v] *= corr;
-        m[g] = mnew;
-      }
-    }
-#pragma unroll
-    for (int it = 0; it < ITERS; ++it) {
-      const int ls = it * SPW + lane_slot;
-      float vf[VEC];
-      Elem<T>::unpack(*reinterpret_cast<const uint4*>(Vs + ls * HD + lane_part * VEC), vf);
-#pragma unroll
-      for (int g = 0; g < G; ++g) {
-        if (sc[g][it] != -INFINITY) {  // masked slots never touch the sums (NaN-safe)
-          const float pr = exp2f(sc[g][it] - m[g]);
-          l[g] += pr;
-#pragma unroll
-          for (int v = 0; v < VEC; ++v) acc[g][v] = fmaf(pr, vf[v], acc[g][v]);
-        }
-      }
-    }
+    if (valid_slots >= STAGE_SLOTS && mask == all_pages)
+      consume_stage<T, HD, G, SB, true>(Ks, Vs, lane_slot, lane_part, q2, p.qscale, valid_slots, mask,
+                                    log2P_in_stage, st);
+    else
+      consume_stage<T, HD, G, SB, false>(Ks, Vs, lane_slot, lane_part, q2, p.qscale, valid_slots, mask,
+                                     log2P_in_stage, st);
     __syncwarp();  // every lane is done with this ring slot
     if (xp < x1) issue(buf);
 
-    const bool end = (x == x1 - 1) || cc.st == cc.nst - 1;
-    if (end) {
-      // merge the lane groups of the warp
+    if ((x == x1 - 1) || cc.st == cc.nst - 1) {
+      // merge the SPW lane groups of the warp
 #pragma unroll
       for (int g = 0; g < G; ++g) {
-        float M = m[g];
+        float M = st.m[g];
 #pragma unroll
-        for (int o = LPS; o < 32; o <<= 1) M = fmaxf(M, __shfl_xor_sync(0xFFFFFFFFu, M, o));
-        const float w = (m[g] == -INFINITY) ? 0.f : exp2f(m[g] - M);
-        float Ls = l[g] * w;
+        for (int o = LPS; o < 32; o <<= 1) M = fmaxf(M, __shfl_xor_sync(FULLMASK, M, o));
+        const float w = (st.m[g] == -INFINITY) ? 0.f : exp2f(st.m[g] - M);
+        float Ls = st.l[g] * w;
 #pragma unroll
-        for (int o = LPS; o < 32; o <<= 1) Ls += __shfl_xor_sync(0xFFFFFFFFu, Ls, o);
+        for (int o = LPS; o < 32; o <<= 1) Ls += __shfl_xor_sync(FULLMASK, Ls, o);
 #pragma unroll
-        for (int v = 0; v < VEC; ++v) {
-          float a = acc[g][v] * w;
+        for (int i = 0; i < E2; ++i) {
+          float2 a = __fmul2_rn(st.acc[g][i], make_float2(w, w));
 #pragma unroll
-          for (int o = LPS; o < 32; o <<= 1) a += __shfl_xor_sync(0xFFFFFFFFu, a, o);
-          acc[g][v] = a;
+          for (int o = LPS; o < 32; o <<= 1) {
+            a.x += __shfl_xor_sync(FULLMASK, a.x, o);
+            a.y += __shfl_xor_sync(FULLMASK, a.y, o);
+          }
+          st.acc[g][i] = a;
         }
-        m[g] = M;
-        l[g] = Ls;
+        st.m[g] = M;
+        st.l[g] = Ls;
       }
       const int64_t rowbase = (int64_t)cc.b * p.Hq + cc.h * G;
       const int64_t U = (int64_t)Hkv * pre[cc.b] + (int64_t)cc.h * cc.nst;
       const int64_t g_first = warp_of(U, NS, GW), g_last = warp_of(U + cc.nst - 1, NS, GW);
       T* outp = reinterpret_cast<T*>(p.out);
       if (g_first == g_last) {
-        if (lane_slot == 0) {
-#pragma unroll
-          for (int g = 0; g < G; ++g) {
-            float o[VEC];
-            const float inv = l[g] > 0.f ? 1.f / l[g] : 0.f;
-#pragma unroll
-            for (int v = 0; v < VEC; ++v) o[v] = acc[g][v] * inv;
-            store_vec<T>(outp + (rowbase + g) * HD + lane_part * VEC, o);
-          }
-        }
+        if (lane_slot == 0) write_rows<T, HD, G, SB>(outp + rowbase * HD, lane_part, st);
       } else {
-        // partial of this piece: its warp's first piece -> A[gw], last piece -> Z[gw]
+        // partial of this piece: its warp's first piece -> side 0, last piece -> side 1
         const bool is_last_piece = (x == x1 - 1);
         for (int side = 0; side < 2; ++side) {
           if ((side == 0 && !piece_first) || (side == 1 && !is_last_piece)) continue;
@@ -365,13 +448,17 @@ __global__ void __launch_bounds__(kThreads) decode_attn_kernel(const AttnParams 
 #pragma unroll
             for (int g = 0; g < G; ++g)
 #pragma unroll
-              for (int v = 0; v < VEC; ++v) po[g * HD + lane_part * VEC + v] = acc[g][v];
+              for (int v = 0; v < SH::NVL; ++v)
+#pragma unroll
+                for (int i = 0; i < VEC / 2; ++i)
+                  reinterpret_cast<float2*>(po + g * HD + (v * LPS + lane_part) * VEC)[i] =
+                      st.acc[g][v * VEC / 2 + i];
           }
           if (lane == 0) {
 #pragma unroll
             for (int g = 0; g < G; ++g) {
-              pm[2 * g] = m[g];
-              pm[2 * g + 1] = l[g];
+              pm[2 * g] = st.m[g];
+              pm[2 * g + 1] = st.l[g];
             }
           }
         }
@@ -382,30 +469,48 @@ __global__ void __launch_bounds__(kThreads) decode_attn_kernel(const AttnParams 
           const int t = atomicAdd(&p.counters[cc.b * Hkv + cc.h], 1);
           last = (t == (int)(g_last - g_first));
         }
-        last = __shfl_sync(0xFFFFFFFFu, last, 0);
+        last = __shfl_sync(FULLMASK, last, 0);
         if (last) {
           __threadfence();
-          // merge pieces of warps g_first .. g_last (Z of the first, A of the rest)
+          // merge the pieces of warps g_first .. g_last (side 1 of the first warp,
+          // side 0 of the others), up to 32 pieces per round, one per lane
+          const int np = (int)(g_last - g_first + 1);
           for (int g = 0; g < G; ++g) {
-            float M = -INFINITY;
-            for (int64_t q = g_first; q <= g_last; ++q) {
-              const int side = q == g_first ? 1 : 0;
-              M = fmaxf(M, __ldcg(p.part_ml + ((int64_t)side * p.nwarps + q) * G * 2 + 2 * g));
-            }
+            float M = -INFINITY, Ls = 0.f;
             float o[HD / 32];
 #pragma unroll
             for (int i = 0; i < HD / 32; ++i) o[i] = 0.f;
-            float Ls = 0.f;
-            for (int64_t q = g_first; q <= g_last; ++q) {
-              const int side = q == g_first ? 1 : 0;
-              const float* pm = p.part_ml + ((int64_t)side * p.nwarps + q) * G * 2 + 2 * g;
-              const float mq = __ldcg(pm);
-              if (mq == -INFINITY) continue;
-              const float w = exp2f(mq - M);
-              Ls = fmaf(w, __ldcg(pm + 1), Ls);
-              const float* po = p.part_o + (((int64_t)side * p.nwarps + q) * G + g) * HD;
+            for (int r0 = 0; r0 < np; r0 += 32) {
+              const int nr = min(32, np - r0);
+              float mq = -INFINITY, lq = 0.f;
+              if (lane < nr) {
+                const int64_t q = g_first + r0 + lane;
+                const float* pm = p.part_ml + ((int64_t)(q == g_first ? 1 : 0) * p.nwarps + q) * G * 2 + 2 * g;
+                mq = __ldcg(pm);
+                lq = __ldcg(pm + 1);
+              }
+              float Mr = mq;
 #pragma unroll
-              for (int i = 0; i < HD / 32; ++i) o[i] = fmaf(w, __ldcg(po + lane + 32 * i), o[i]);
+              for (int o2 = 16; o2 > 0; o2 >>= 1) Mr = fmaxf(Mr, __shfl_xor_sync(FULLMASK, Mr, o2));
+              const float Mn = fmaxf(M, Mr);
+              if (Mn == -INFINITY) continue;
+              const float rescale = exp2f(M - Mn);  // 0 on the first round
+              const float w = (mq == -INFINITY) ? 0.f : exp2f(mq - Mn);
+              float lw = w * lq;
+#pragma unroll
+              for (int o2 = 16; o2 > 0; o2 >>= 1) lw += __shfl_xor_sync(FULLMASK, lw, o2);
+              Ls = Ls * rescale + lw;
+#pragma unroll
+              for (int i = 0; i < HD / 32; ++i) o[i] *= rescale;
+#pragma unroll 4
+              for (int j = 0; j < nr; ++j) {
+                const float wj = __shfl_sync(FULLMASK, w, j);
+                const int64_t q = g_first + r0 + j;
+                const float* po = p.part_o + (((int64_t)(q == g_first ? 1 : 0) * p.nwarps + q) * G + g) * HD;
+#pragma unroll
+                for (int i = 0; i < HD / 32; ++i) o[i] = fmaf(wj, __ldcg(po + lane + 32 * i), o[i]);
+              }
+              M = Mn;
             }
             const float inv = Ls > 0.f ? 1.f / Ls : 0.f;
 #pragma unroll
@@ -421,59 +526,69 @@ __global__ void __launch_bounds__(kThreads) decode_attn_kernel(const AttnParams 
   }
 }
 
-template <typename T, int HD>
-constexpr int stage_slots() {
-  return Shape<T, HD>::STAGE_SLOTS;
-}
-
-template <typename T, int HD, int G>
+template <typename T, int HD, int G, int SB>
 cudaError_t launch_t(const AttnParams& p, int grid, size_t smem, cudaStream_t stream) {
   static size_t smem_set = 0;  // largest dynamic smem opted into so far
-  auto kern = decode_attn_kernel<T, HD, G>;
+  auto kern = decode_attn_kernel<T, HD, G, SB>;
   if (smem > smem_set) {
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     smem_set = smem;
   }
-  kern<<<grid, kThreads, smem, stream>>>(p);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, p);
 }
 
-template <typename T, int HD>
+template <typename T, int HD, int SB>
 cudaError_t launch_g(const AttnParams& p, int G, int grid, size_t smem, cudaStream_t s) {
   switch (G) {
-    case 1: return launch_t<T, HD, 1>(p, grid, smem, s);
-    case 2: return launch_t<T, HD, 2>(p, grid, smem, s);
-    case 4: return launch_t<T, HD, 4>(p, grid, smem, s);
-    case 8: return launch_t<T, HD, 8>(p, grid, smem, s);
+    case 1: return launch_t<T, HD, 1, SB>(p, grid, smem, s);
+    case 2: return launch_t<T, HD, 2, SB>(p, grid, smem, s);
+    case 4: return launch_t<T, HD, 4, SB>(p, grid, smem, s);
+    case 8: return launch_t<T, HD, 8, SB>(p, grid, smem, s);
     default: return cudaErrorInvalidValue;
   }
 }
 
+template <int SB>
+cudaError_t launch_sb(const AttnParams& p, int dtype, int d, int G, int grid, size_t smem,
+                      cudaStream_t s) {
+  if (dtype == WM_DT_F32)
+    return d == 64 ? launch_g<float, 64, SB>(p, G, grid, smem, s)
+                   : launch_g<float, 128, SB>(p, G, grid, smem, s);
+  return d == 64 ? launch_g<__nv_bfloat16, 64, SB>(p, G, grid, smem, s)
+                 : launch_g<__nv_bfloat16, 128, SB>(p, G, grid, smem, s);
+}
+
 }  // namespace
 
-int attn_stage_slots(int dtype, int d) {
-  if (dtype == WM_DT_F32) return d == 64 ? stage_slots<float, 64>() : stage_slots<float, 128>();
-  return d == 64 ? stage_slots<__nv_bfloat16, 64>() : stage_slots<__nv_bfloat16, 128>();
+int attn_stage_slots(int stage_bytes, int dtype, int d) {
+  return stage_bytes / (2 * d * (dtype == WM_DT_F32 ? 4 : 2));
 }
 
 int attn_warps_per_cta() { return kWarps; }
 
-size_t attn_smem_bytes(int dtype, int d, int G, int B) {
+size_t attn_smem_bytes(int stage_bytes, int dtype, int d, int G, int B) {
   const size_t esz = dtype == WM_DT_F32 ? 4 : 2;
-  return (size_t)kWarps * kWStages * kWStageBytes + (size_t)kWarps * kWStages * G * d * esz +
+  return (size_t)kWarps * kWStages * stage_bytes + (size_t)kWarps * kWStages * G * d * esz +
          sizeof(int) * (2 * (size_t)B + 1);
 }
 
-cudaError_t launch_decode_attn(const AttnParams& p, int dtype, int d, int G, int grid,
-                               cudaStream_t s) {
-  const size_t smem = attn_smem_bytes(dtype, d, G, p.B);
-  if (dtype == WM_DT_F32) {
-    return d == 64 ? launch_g<float, 64>(p, G, grid, smem, s)
-                   : launch_g<float, 128>(p, G, grid, smem, s);
-  }
-  return d == 64 ? launch_g<__nv_bfloat16, 64>(p, G, grid, smem, s)
-                 : launch_g<__nv_bfloat16, 128>(p, G, grid, smem, s);
+cudaError_t launch_decode_attn(const AttnParams& p, int stage_bytes, int dtype, int d, int G,
+                               int grid, cudaStream_t s) {
+  const size_t smem = attn_smem_bytes(stage_bytes, dtype, d, G, p.B);
+  if (stage_bytes == 4096) return launch_sb<4096>(p, dtype, d, G, grid, smem, s);
+  if (stage_bytes == 8192) return launch_sb<8192>(p, dtype, d, G, grid, smem, s);
+  return cudaErrorInvalidValue;
 }
 
 }  // namespace wm

@@ -26,11 +26,11 @@ struct AttnParams {
   float qscale;           // log2(e) / sqrt(d)
 };
 
-int attn_stage_slots(int dtype, int d);
+int attn_stage_slots(int stage_bytes, int dtype, int d);
 int attn_warps_per_cta();
-size_t attn_smem_bytes(int dtype, int d, int G, int B);
-cudaError_t launch_decode_attn(const AttnParams& p, int dtype, int d, int G, int grid,
-                               cudaStream_t s);
+size_t attn_smem_bytes(int stage_bytes, int dtype, int d, int G, int B);
+cudaError_t launch_decode_attn(const AttnParams& p, int stage_bytes, int dtype, int d, int G,
+                               int grid, cudaStream_t s);
 
 // ------------------------------------------------------------ KV pool (mix)
 constexpr int kMaxRopeHalf = 64;  // d/2 for d <= 128

@@ -34,21 +34,27 @@ bool aligned(const void* p, size_t a) { return ((uintptr_t)p % a) == 0; }
 
 // Persistent grid of one attention launch and its workspace layout.
 struct AttnPlan {
-  int grid, nwarps;
+  int stage_bytes, grid, nwarps;
   size_t off_part_o, off_part_ml, off_counters, total;
 };
 
-constexpr int kAttnCtasPerSm = 2;
 constexpr int kAttnMaxBatch = 4096;
+// Launches reading less than this many KV bytes (upper bound from the page
+// table width) use 4 KB stages and 4 CTAs per SM (16 warps: more latency
+// hiding for short launches); larger ones use 8 KB stages and 2 CTAs per SM.
+constexpr double kAttnSmallLaunchBytes = 1.0e9;
 
 AttnPlan attn_plan(const wm_config& c, int32_t B, int32_t max_pages) {
   AttnPlan pl{};
-  const int stage = wm::attn_stage_slots(c.dtype, c.d);
   const int64_t max_slots = (int64_t)max_pages * c.page_size;
+  const double kv_bytes = (double)B * c.Hkv * max_slots * 2.0 * c.d * elem_size(c.dtype);
+  pl.stage_bytes = kv_bytes < kAttnSmallLaunchBytes ? 4096 : 8192;
+  const int ctas_per_sm = pl.stage_bytes == 4096 ? 4 : 2;
+  const int stage = wm::attn_stage_slots(pl.stage_bytes, c.dtype, c.d);
   const int64_t ns_max = (int64_t)B * c.Hkv * ((max_slots + stage - 1) / stage);
   const int wpc = wm::attn_warps_per_cta();
-  // one CTA pair per SM, fewer when there are under 4 stages per warp
-  int64_t grid = (int64_t)sm_count() * kAttnCtasPerSm;
+  // fill the SMs, but keep at least 4 stages per warp
+  int64_t grid = (int64_t)sm_count() * ctas_per_sm;
   const int64_t by_work = (ns_max + 4 * wpc - 1) / (4 * wpc);
   if (by_work < grid) grid = by_work;
   if (grid < 1) grid = 1;
@@ -180,8 +186,8 @@ wm_status wm_decode_attn(const wm_config* c, const wm_cache* cache, int32_t laye
   p.B = B;
   p.nwarps = pl.nwarps;
   p.qscale = (float)(1.4426950408889634 / sqrt((double)c->d));
-  cudaError_t e = wm::launch_decode_attn(p, c->dtype, c->d, c->Hq / c->Hkv, pl.grid,
-                                         (cudaStream_t)stream);
+  cudaError_t e = wm::launch_decode_attn(p, pl.stage_bytes, c->dtype, c->d, c->Hq / c->Hkv,
+                                         pl.grid, (cudaStream_t)stream);
   return e == cudaSuccess ? WM_OK : WM_ERR_CUDA;
 }
 

@@ -181,6 +181,39 @@ wm_status wm_decode_attn(const wm_config* cfg, const wm_cache* cache, int32_t la
                          int32_t B, int32_t max_pages, void* out, void* workspace,
                          size_t ws_bytes, int32_t* dev_status, void* stream);
 
+/*
+ * Decode attention for callers that cannot allocate device memory.
+ *
+ * The paper has no counterpart: this is a deployment variant of
+ * wm_decode_attn.  Some callers cannot provide the workspace that
+ * wm_decode_attn asks for: for example a plugin running inside a host
+ * program whose allocator owns all device memory and does not let it
+ * allocate, or a caller working to a fixed memory plan with no room for
+ * scratch.  This entry point computes exactly what wm_decode_attn computes,
+ * with the same arguments minus the workspace, and allocates nothing: its
+ * scratch is a fixed array of WM_NOALLOC_SCRATCH_BYTES bytes inside the
+ * library's device image, which every GPU that loads the library keeps
+ * until the process exits.
+ *
+ *  - The first call on a device looks up that array's device address
+ *    (cudaGetSymbolAddress) with the device current; make that first call
+ *    before any stream capture.
+ *  - Each call clears the part of the array that must start at zero (the
+ *    arrival tickets) with an asynchronous memset on `stream`, then launches.
+ *  - All calls in the process share the one array per device: calls that
+ *    overlap on the GPU (different streams without ordering) race and give
+ *    wrong results.  Serialise them, e.g. on one stream.
+ *  - Returns WM_ERR_UNSUPPORTED when the launch would need more scratch than
+ *    WM_NOALLOC_SCRATCH_BYTES (large batch x heads x group sizes); use
+ *    wm_decode_attn with a workspace then.  Other errors as wm_decode_attn.
+ */
+#define WM_NOALLOC_SCRATCH_BYTES (8u << 20)
+
+wm_status wm_decode_attn_noalloc(const wm_config* cfg, const wm_cache* cache, int32_t layer,
+                                 const void* q, const int32_t* page_table,
+                                 const int32_t* seq_lens, int32_t B, int32_t max_pages,
+                                 void* out, int32_t* dev_status, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

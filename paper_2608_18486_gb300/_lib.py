@@ -153,3 +153,18 @@ def wm_decode_attn(cfg, cache, layer, q, page_table, seq_lens, B, max_pages, out
     return lib().wm_decode_attn(ctypes.byref(cfg), ctypes.byref(cache), int(layer), _p(q),
                                 _p(page_table), _p(seq_lens), int(B), int(max_pages), _p(out),
                                 _p(workspace), int(ws_bytes), _p(dev_status), stream)
+
+
+def wm_decode_attn_noalloc(cfg, cache, layer, q, page_table, seq_lens, B, max_pages, out,
+                           dev_status, stream) -> int:
+    """Decode attention with the library's own fixed scratch (no workspace)."""
+    L = lib()
+    if not getattr(L, "_noalloc_typed", False):
+        cp, vp, i32 = ctypes.POINTER(wm_config), ctypes.c_void_p, ctypes.c_int32
+        L.wm_decode_attn_noalloc.restype = ctypes.c_int
+        L.wm_decode_attn_noalloc.argtypes = [cp, ctypes.POINTER(wm_cache), i32, vp, vp, vp, i32,
+                                             i32, vp, vp, vp]
+        L._noalloc_typed = True
+    return L.wm_decode_attn_noalloc(ctypes.byref(cfg), ctypes.byref(cache), int(layer), _p(q),
+                                    _p(page_table), _p(seq_lens), int(B), int(max_pages), _p(out),
+                                    _p(dev_status), stream)

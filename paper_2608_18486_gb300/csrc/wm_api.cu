@@ -3,6 +3,8 @@
 #include <math.h>
 #include <string.h>
 
+#include <mutex>
+
 #include "internal.h"
 #include "wm.h"
 
@@ -262,3 +264,60 @@ wm_status wm_kv_mix(const wm_config* c, const wm_cache* cache, const wm_mix_weig
 }
 
 }  // extern "C"
+
+// ------------------------------------------------------------------------
+// Decode attention without caller-provided scratch.
+//
+// Some callers cannot hand this library any device memory beyond the inputs
+// and outputs of a call: a plugin inside a host program whose allocator owns
+// the whole device and forbids other allocations, or a caller with a fixed
+// memory plan that has no room for a workspace.  For them the attention's
+// scratch (per-warp partial results and arrival tickets) lives in one
+// fixed-size array that is part of this library's device image.  Every GPU
+// that loads the library holds the array until the process exits.
+namespace {
+
+static __device__ __align__(256) unsigned char g_noalloc_scratch[WM_NOALLOC_SCRATCH_BYTES];
+
+std::mutex g_noalloc_mu;
+void* g_noalloc_ptr[kMaxDevices];  // device address of the array, per device
+
+// Device address of the array on the current device.  Host code cannot use
+// the symbol itself (it names a host-side stand-in), so the address is asked
+// for once per device, with that device current.
+wm_status noalloc_scratch(void** out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return WM_ERR_CUDA;
+  std::lock_guard<std::mutex> lock(g_noalloc_mu);
+  if (!g_noalloc_ptr[dev]) {
+    void* ptr = nullptr;
+    if (cudaGetSymbolAddress(&ptr, g_noalloc_scratch) != cudaSuccess || !ptr) return WM_ERR_CUDA;
+    g_noalloc_ptr[dev] = ptr;
+  }
+  *out = g_noalloc_ptr[dev];
+  return WM_OK;
+}
+
+}  // namespace
+
+extern "C" wm_status wm_decode_attn_noalloc(const wm_config* c, const wm_cache* cache,
+                                            int32_t layer, const void* q,
+                                            const int32_t* page_table, const int32_t* seq_lens,
+                                            int32_t B, int32_t max_pages, void* out,
+                                            int32_t* dev_status, void* stream) {
+  wm_status st = wm_config_check(c);
+  if (st != WM_OK) return st;
+  if (B < 0 || max_pages < 1) return WM_ERR_INVALID_ARG;
+  if (B == 0) return WM_OK;
+  if (B > kAttnMaxBatch) return WM_ERR_UNSUPPORTED;
+  const AttnPlan pl = attn_plan(*c, B, max_pages);
+  if (pl.total > (size_t)WM_NOALLOC_SCRATCH_BYTES) return WM_ERR_UNSUPPORTED;
+  void* scratch = nullptr;
+  if ((st = noalloc_scratch(&scratch)) != WM_OK) return st;
+  // the arrival tickets must start at zero; the array keeps the last call's bytes
+  if (cudaMemsetAsync((char*)scratch + pl.off_counters, 0, pl.total - pl.off_counters,
+                      (cudaStream_t)stream) != cudaSuccess)
+    return WM_ERR_CUDA;
+  return wm_decode_attn(c, cache, layer, q, page_table, seq_lens, B, max_pages, out, scratch,
+                        (size_t)WM_NOALLOC_SCRATCH_BYTES, dev_status, stream);
+}

@@ -118,6 +118,24 @@ class ClockSampler:
                 "samples": len(inside)}
 
 
+def rank_problem(w, rank: int):
+    """The batch of sequences replica `rank` decodes: its own seeded problem
+    (own cache contents, lengths and page table), so ranks share nothing."""
+    from wm_synth.inputs import make_problem
+    return make_problem(w, seed=rank)
+
+
+def max_over_ranks(values, world: int, device=None):
+    """Element-wise max of per-rank timings (the job is as slow as its
+    slowest replica); a no-op for one rank."""
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor(list(values), dtype=torch.float64, device=device)
+    if world > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return [float(x) for x in t]
+
+
 # ---------------------------------------------------------------- CPU oracle timing
 def oracle_step_estimate(prob, budget_s: float = 4.0, nthreads: int | None = None):
     """Time the fp64 oracle on a bounded sample of one decode step and
@@ -230,9 +248,8 @@ def run_gpu(args, w):
     from paper_2608_18486_gb300.session import DecodeSession
     from wm_synth import configs as C
     from wm_synth.device_problem import DeviceProblem
-    from wm_synth.inputs import make_problem
 
-    prob = make_problem(w, seed=rank)  # each replica decodes its own sequences
+    prob = rank_problem(w, rank)  # each replica decodes its own sequences
     cfg = make_config(w.L, w.k, w.D, w.Hq, w.Hkv, w.d, w.p, w.page, w.dtype, w.chan_of_layer(),
                       w.eps_rms, w.eps_qk, w.rope_theta)
     sess = DecodeSession(cfg, w.B, prob.num_pages, prob.max_pages, dev)
@@ -287,10 +304,7 @@ def run_gpu(args, w):
         raise RuntimeError(f"device status {status} during the timed region")
     ms = start.elapsed_time(end)
     attn_ms = sum(a.elapsed_time(b) for a, b in ev)
-    t = torch.tensor([ms, attn_ms], dtype=torch.float64, device=dev)
-    if world > 1:
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-    ms, attn_ms = float(t[0]), float(t[1])
+    ms, attn_ms = max_over_ranks([ms, attn_ms], world, dev)
 
     # ---- end to end through the public API with pinned host buffers
     q_host = torch.empty(dp.q.shape, dtype=dp.q.dtype, pin_memory=True)
@@ -316,11 +330,7 @@ def run_gpu(args, w):
             e2e_step()
     e_end.record(stream)
     barrier()
-    e2e_ms = e_start.elapsed_time(e_end)
-    te = torch.tensor([e2e_ms], dtype=torch.float64, device=dev)
-    if world > 1:
-        dist.all_reduce(te, op=dist.ReduceOp.MAX)
-    e2e_ms = float(te[0])
+    e2e_ms = max_over_ranks([e_start.elapsed_time(e_end)], world, dev)[0]
 
     if rank == 0:
         tokens = w.B * world * args.steps
@@ -368,9 +378,17 @@ def main():
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--ref-budget", type=float, default=4.0,
                     help="seconds of oracle time per reference/CPU-baseline sample")
+    ap.add_argument("--set", action="append", default=[], metavar="FIELD=VALUE",
+                    help="override a workload field, e.g. --set k=1 (smaller cache for profiling)")
     args = ap.parse_args()
     from wm_synth import configs
     w = configs.get(args.workload)
+    for kv in args.set:
+        key, val = kv.split("=", 1)
+        cur = getattr(w, key)
+        w = w.with_(**{key: type(cur)(val) if not isinstance(cur, bool) else val == "1"})
+    if args.set:
+        w = w.with_(name=w.name + "[" + ",".join(args.set) + "]")
     if args.warmup < 3 and args.impl != "reference":
         args.warmup = 3
     if args.impl == "reference":

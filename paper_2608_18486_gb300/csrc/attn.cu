@@ -6,21 +6,23 @@
 // per FLOP, so it is HBM-bound and runs on the CUDA cores.
 //
 //  * Stream-K split.  Each unit is cut into pipeline stages of STAGE_SLOTS
-//    slots (8 KB of K+V).  The stages of all units, concatenated, are divided
-//    into equal contiguous ranges, one per warp of a persistent grid, so every
-//    warp streams the same number of bytes whatever the sequence lengths.
+//    slots (4 or 8 KB of K+V).  The stages of all units, concatenated, are
+//    cut into equal chunks of CH stages.  Warp w of the persistent grid
+//    starts on chunk w and then takes further chunks from an atomic counter
+//    (requested one chunk ahead), so warps that stream faster take more
+//    chunks and all finish together whatever the sequence lengths.
 //  * Private pipelines.  Each warp owns a 3-deep ring in shared memory and
 //    fills it with 1-D bulk async copies (TMA engine, mbarrier completion,
 //    L2 evict-first) of contiguous (page, kv-head) runs; it refills a slot as
 //    soon as it has consumed it, so no block-wide barrier is ever taken.
-//  * Compute.  d/VEC lanes own one slot (a 16-byte vector each), reduce q.k
-//    with xor shuffles and keep an online softmax (running max m, sum l,
-//    accumulator) per lane group; groups merge with shuffles at the end of a
-//    piece.
-//  * Merge.  A piece of a unit that lies inside one warp's range is written
-//    straight to the output.  Only units that cross a warp boundary leave
-//    partials (at most two per warp: its first and its last piece); the last
-//    warp to finish such a unit (atomic ticket, no waiting) merges them.
+//  * Compute.  8 lanes own one slot (16-byte vectors, conflict-free shared
+//    loads), reduce q.k with xor shuffles and keep an online softmax
+//    (running max m, sum l, accumulator) per lane group; groups merge with
+//    shuffles at the end of a piece.
+//  * Merge.  A piece of a unit that lies inside one chunk is written straight
+//    to the output.  Only units that cross a chunk boundary leave partials
+//    (at most two per chunk: its first and its last piece); the last warp to
+//    finish such a unit (atomic ticket, no waiting) merges them.
 #include <math.h>
 
 #include "common.cuh"
@@ -110,10 +112,6 @@ __device__ __forceinline__ void advance(Cursor& c, const int* pre, int B, int Hk
   if (c.b < B) c.nst = pre[c.b + 1] - pre[c.b];
 }
 
-// Warp owning global stage x: the largest g with floor(g * NS / GW) <= x.
-__device__ __forceinline__ int64_t warp_of(int64_t x, int64_t NS, int64_t GW) {
-  return ((x + 1) * GW - 1) / NS;
-}
 
 // Online-softmax state of one lane: G query heads, EPL output elements each.
 template <typename T, int HD, int G, int SB>
@@ -270,13 +268,39 @@ __global__ void __launch_bounds__(kThreads, SB == 4096 ? 4 : 2) decode_attn_kern
     }
   }
 
-  // Equal stage ranges over the first GW warps; with fewer stages than warps
-  // only NS warps take one stage each, so every warp in a unit's span has work.
-  const int64_t NS = (int64_t)Hkv * pre[B];
-  const int64_t GW = min((int64_t)gridDim.x * kWarps, NS);
+  // The NS stages split into nchunks near-equal chunks [c*NS/n, (c+1)*NS/n).
+  // Every chunk has at least CH > kWStages stages, so the producer, at most
+  // kWStages stages ahead, is never more than one chunk ahead of the consumer.
+  // chunk_stages == 0: static split, one chunk per warp and no chunk counter.
+  const int64_t NS = (int64_t)Hkv * pre[B];  // stages of all units, concatenated
+  const int64_t GW = (int64_t)gridDim.x * kWarps;
+  const bool dynamic = p.chunk_stages > 0;
+  const int64_t CH = dynamic ? p.chunk_stages : (int64_t)kWStages + 1;
+  int64_t nchunks = NS / CH > 1 ? NS / CH : 1;
+  if (!dynamic && nchunks > GW) nchunks = GW;
+  auto chunk_begin = [&](int64_t c) -> int64_t { return c * NS / nchunks; };
+  auto chunk_end_x = [&](int64_t c) -> int64_t { return (c + 1) * NS / nchunks; };
+  auto chunk_of = [&](int64_t x) -> int64_t { return ((x + 1) * nchunks - 1) / NS; };
   const int64_t gw = (int64_t)blockIdx.x * kWarps + warp;
-  if (gw >= GW) return;  // warp-level from here on: no block barriers below
-  const int64_t x0 = gw * NS / GW, x1 = (gw + 1) * NS / GW;
+  int32_t* grab_ctr = p.counters + (int64_t)B * Hkv;
+  // Every warp ends with exactly one request that finds no chunk; the request
+  // that is last of all resets the counter for the next launch.  A request is
+  // issued one chunk ahead and its result read only when the chunk is needed.
+  const int64_t total_grabs = (nchunks > GW ? nchunks - GW : 0) + GW;
+  int grab_t = 0;  // lane 0: counter value of the outstanding request
+  auto grab_issue = [&]() {
+    if (dynamic && lane == 0) grab_t = atomicAdd(grab_ctr, 1);
+  };
+  auto grab_take = [&]() -> int64_t {
+    if (!dynamic) return nchunks;  // static split: no further chunk
+    if (lane == 0 && grab_t == total_grabs - 1) atomicExch(grab_ctr, 0);
+    return GW + __shfl_sync(FULLMASK, grab_t, 0);
+  };
+  if (gw >= nchunks || NS == 0) {
+    grab_issue();
+    grab_take();
+    return;  // warp-level from here on: no block barriers below
+  }
 
   T* myring = ring + warp * kWStages * 2 * STAGE_ELEMS;
   T* myq = qring + warp * kWStages * G * HD;
@@ -307,11 +331,17 @@ __global__ void __launch_bounds__(kThreads, SB == 4096 ? 4 : 2) decode_attn_kern
     return idx < 32 ? a : c;
   };
 
-  // ---- producer: stage xp at cursor pc into ring slot buf
-  Cursor pc = locate(x0, pre, B, Hkv);
-  int64_t xp = x0;
-  auto issue = [&](int buf) {
-    const bool first = (xp == x0) || pc.st == 0;
+  // ---- producer: walks its chunks stage by stage, kWStages ahead of the consumer
+  int64_t p_chunk = gw;
+  grab_issue();                                 // the next chunk, requested one ahead
+  int64_t px = chunk_begin(p_chunk), pend = chunk_end_x(p_chunk);
+  int64_t chunk_for_consumer = -1;              // the producer's chunk after a switch
+  bool p_done = false;
+  Cursor pc = locate(px, pre, B, Hkv);
+  uint32_t pseq = 0;                            // stages issued
+  auto issue = [&]() {
+    const int buf = (int)(pseq % kWStages);
+    const bool first = (px == chunk_begin(p_chunk)) || pc.st == 0;
     const int S = lens[pc.b];
     const int s_begin = pc.st * STAGE_SLOTS;
     const T* kb = reinterpret_cast<const T*>(p.k_pool) + (int64_t)pc.h * p.P * HD;
@@ -356,34 +386,48 @@ __global__ void __launch_bounds__(kThreads, SB == 4096 ? 4 : 2) decode_attn_kern
         bulk_g2s(vd + lane * p.P * HD, vb + off, bytes, bar, policy);
       }
     }
-    ++xp;
+    ++pseq;
+    ++px;
     advance(pc, pre, B, Hkv);
+    if (px == pend) {  // chunk finished: move to the chunk requested ahead
+      p_chunk = grab_take();
+      chunk_for_consumer = p_chunk;
+      if (p_chunk < nchunks) {
+        px = chunk_begin(p_chunk);
+        pend = chunk_end_x(p_chunk);
+        pc = locate(px, pre, B, Hkv);
+        grab_issue();
+      } else {
+        p_done = true;
+      }
+    }
   };
 
-  for (int s = 0; s < kWStages && xp < x1; ++s) issue(s);
+  for (int s = 0; s < kWStages && !p_done; ++s) issue();
 
   // ---- consumer
   const int log2P_in_stage = p.P >= STAGE_SLOTS ? 30 : p.log2P;  // stage page index = slot >> this
   const uint64_t all_pages = p.P >= STAGE_SLOTS ? 1ull : ((1ull << (STAGE_SLOTS >> p.log2P)) - 1ull);
-  Cursor cc = locate(x0, pre, B, Hkv);
-  bool piece_first = true;  // the piece that starts at x0 is this warp's first
+  int64_t c_chunk = gw;
+  int64_t cx = chunk_begin(c_chunk), cend = chunk_end_x(c_chunk);
+  Cursor cc = locate(cx, pre, B, Hkv);
+  bool piece_first = true;  // the current piece starts at its chunk's first stage
   float2 q2[G][E2];
   SoftState<T, HD, G, SB> st;
-  for (int64_t x = x0; x < x1; ++x) {
-    const int buf = (int)((x - x0) % kWStages);
-    const uint32_t parity = (uint32_t)(((x - x0) / kWStages) & 1);
-    const bool ok = mbar_wait(&bars[warp][buf], parity);
+  T* outp = reinterpret_cast<T*>(p.out);
+  for (uint32_t seq = 0;; ++seq) {
+    const int buf = (int)(seq % kWStages);
+    const bool ok = mbar_wait(&bars[warp][buf], (seq / kWStages) & 1);
     if (__any_sync(FULLMASK, !ok)) {
       // a copy never landed: report, drain what is in flight (bounded) and stop
       if (lane == 0) {
         report(p.status, WM_ERR_TIMEOUT);
-        for (int64_t y = x; y < xp; ++y)
-          mbar_wait(&bars[warp][(y - x0) % kWStages], (uint32_t)(((y - x0) / kWStages) & 1));
+        for (uint32_t y = seq; y < pseq; ++y) mbar_wait(&bars[warp][y % kWStages], (y / kWStages) & 1);
       }
       __syncwarp();
       return;
     }
-    if ((x == x0) || cc.st == 0) {
+    if (cx == chunk_begin(c_chunk) || cc.st == 0) {
       const T* qs = myq + buf * G * HD;
 #pragma unroll
       for (int g = 0; g < G; ++g) {
@@ -399,15 +443,16 @@ __global__ void __launch_bounds__(kThreads, SB == 4096 ? 4 : 2) decode_attn_kern
     const T* Ks = myring + buf * 2 * STAGE_ELEMS;
     const T* Vs = Ks + STAGE_ELEMS;
     if (valid_slots >= STAGE_SLOTS && mask == all_pages)
-      consume_stage<T, HD, G, SB, true>(Ks, Vs, lane_slot, lane_part, q2, p.qscale, valid_slots, mask,
-                                    log2P_in_stage, st);
+      consume_stage<T, HD, G, SB, true>(Ks, Vs, lane_slot, lane_part, q2, p.qscale, valid_slots,
+                                        mask, log2P_in_stage, st);
     else
-      consume_stage<T, HD, G, SB, false>(Ks, Vs, lane_slot, lane_part, q2, p.qscale, valid_slots, mask,
-                                     log2P_in_stage, st);
+      consume_stage<T, HD, G, SB, false>(Ks, Vs, lane_slot, lane_part, q2, p.qscale, valid_slots,
+                                         mask, log2P_in_stage, st);
     __syncwarp();  // every lane is done with this ring slot
-    if (xp < x1) issue(buf);
+    if (!p_done) issue();
 
-    if ((x == x1 - 1) || cc.st == cc.nst - 1) {
+    const bool chunk_end = (cx == cend - 1);
+    if (chunk_end || cc.st == cc.nst - 1) {
       // merge the SPW lane groups of the warp
 #pragma unroll
       for (int g = 0; g < G; ++g) {
@@ -433,17 +478,15 @@ __global__ void __launch_bounds__(kThreads, SB == 4096 ? 4 : 2) decode_attn_kern
       }
       const int64_t rowbase = (int64_t)cc.b * p.Hq + cc.h * G;
       const int64_t U = (int64_t)Hkv * pre[cc.b] + (int64_t)cc.h * cc.nst;
-      const int64_t g_first = warp_of(U, NS, GW), g_last = warp_of(U + cc.nst - 1, NS, GW);
-      T* outp = reinterpret_cast<T*>(p.out);
+      const int64_t g_first = chunk_of(U), g_last = chunk_of(U + cc.nst - 1);
       if (g_first == g_last) {
         if (lane_slot == 0) write_rows<T, HD, G, SB>(outp + rowbase * HD, lane_part, st);
       } else {
-        // partial of this piece: its warp's first piece -> side 0, last piece -> side 1
-        const bool is_last_piece = (x == x1 - 1);
+        // partial of this piece: its chunk's first piece -> side 0, last piece -> side 1
         for (int side = 0; side < 2; ++side) {
-          if ((side == 0 && !piece_first) || (side == 1 && !is_last_piece)) continue;
-          float* po = p.part_o + ((int64_t)side * p.nwarps + gw) * G * HD;
-          float* pm = p.part_ml + ((int64_t)side * p.nwarps + gw) * G * 2;
+          if ((side == 0 && !piece_first) || (side == 1 && !chunk_end)) continue;
+          float* po = p.part_o + ((int64_t)side * p.max_chunks + c_chunk) * G * HD;
+          float* pm = p.part_ml + ((int64_t)side * p.max_chunks + c_chunk) * G * 2;
           if (lane_slot == 0) {
 #pragma unroll
             for (int g = 0; g < G; ++g)
@@ -472,8 +515,8 @@ __global__ void __launch_bounds__(kThreads, SB == 4096 ? 4 : 2) decode_attn_kern
         last = __shfl_sync(FULLMASK, last, 0);
         if (last) {
           __threadfence();
-          // merge the pieces of warps g_first .. g_last (side 1 of the first warp,
-          // side 0 of the others), up to 32 pieces per round, one per lane
+          // merge the pieces of chunks g_first .. g_last (side 1 of the first
+          // chunk, side 0 of the others), up to 32 pieces per round, one per lane
           const int np = (int)(g_last - g_first + 1);
           for (int g = 0; g < G; ++g) {
             float M = -INFINITY, Ls = 0.f;
@@ -485,7 +528,7 @@ __global__ void __launch_bounds__(kThreads, SB == 4096 ? 4 : 2) decode_attn_kern
               float mq = -INFINITY, lq = 0.f;
               if (lane < nr) {
                 const int64_t q = g_first + r0 + lane;
-                const float* pm = p.part_ml + ((int64_t)(q == g_first ? 1 : 0) * p.nwarps + q) * G * 2 + 2 * g;
+                const float* pm = p.part_ml + ((int64_t)(q == g_first ? 1 : 0) * p.max_chunks + q) * G * 2 + 2 * g;
                 mq = __ldcg(pm);
                 lq = __ldcg(pm + 1);
               }
@@ -506,7 +549,7 @@ __global__ void __launch_bounds__(kThreads, SB == 4096 ? 4 : 2) decode_attn_kern
               for (int j = 0; j < nr; ++j) {
                 const float wj = __shfl_sync(FULLMASK, w, j);
                 const int64_t q = g_first + r0 + j;
-                const float* po = p.part_o + (((int64_t)(q == g_first ? 1 : 0) * p.nwarps + q) * G + g) * HD;
+                const float* po = p.part_o + (((int64_t)(q == g_first ? 1 : 0) * p.max_chunks + q) * G + g) * HD;
 #pragma unroll
                 for (int i = 0; i < HD / 32; ++i) o[i] = fmaf(wj, __ldcg(po + lane + 32 * i), o[i]);
               }
@@ -522,7 +565,17 @@ __global__ void __launch_bounds__(kThreads, SB == 4096 ? 4 : 2) decode_attn_kern
       }
       piece_first = false;
     }
-    advance(cc, pre, B, Hkv);
+    if (chunk_end) {  // continue with the chunk the producer moved on to
+      c_chunk = chunk_for_consumer;
+      if (c_chunk < 0 || c_chunk >= nchunks) break;
+      cx = chunk_begin(c_chunk);
+      cend = chunk_end_x(c_chunk);
+      cc = locate(cx, pre, B, Hkv);
+      piece_first = true;
+    } else {
+      ++cx;
+      advance(cc, pre, B, Hkv);
+    }
   }
 }
 

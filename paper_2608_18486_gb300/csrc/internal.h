@@ -16,13 +16,14 @@ struct AttnParams {
   void* out;              // [B][Hq][d]
   const int32_t* page_table;
   const int32_t* seq_lens;
-  float* part_o;          // [2][nwarps][G][d]: first / last piece partial of each warp
-  float* part_ml;         // [2][nwarps][G][2]: (max, sum) in log2 units
-  int32_t* counters;      // [B*Hkv] arrival tickets, zero between launches
+  float* part_o;          // [2][max_chunks][G][d]: first / last piece partial of each chunk
+  float* part_ml;         // [2][max_chunks][G][2]: (max, sum) in log2 units
+  int32_t* counters;      // [B*Hkv] arrival tickets + 1 chunk counter, zero between launches
   int32_t* status;
   int64_t page_stride;    // elements between consecutive physical pages
   int32_t B, Hq, Hkv, P, log2P, num_pages, max_pages;
-  int32_t nwarps;         // warps of the launch grid
+  int32_t chunk_stages;   // stages per work chunk
+  int32_t max_chunks;     // partial slots per side
   float qscale;           // log2(e) / sqrt(d)
 };
 
@@ -54,7 +55,7 @@ struct MixParams {
   void* v_pool;
   // workspace
   float* inv_rms;                 // [B][L]
-  float* xi;                      // [2][B][Lp*D] router inputs (fp32)
+  void* xi;                       // [2][B][Lp*D] router inputs (dtype of the config)
   float* zpart;                   // [2][nsplit_r][B][k*L] router partial sums
   float* rope_cs;                 // [B][d/2][2] cos, sin at pos = slot - 1
   void* xop;                      // [2][k][B][D] normed channels, dtype
@@ -72,8 +73,12 @@ struct MixWorkspace {
 MixWorkspace mix_workspace_layout(const wm_config& cfg, int32_t B, int sm_count);
 cudaError_t launch_kv_mix(MixParams& p, int dtype, cudaStream_t s);
 
-// tcgen05 projection with the fused key/value epilogue (bf16 only)
+// tcgen05 projection with the fused key/value epilogue, and the tcgen05
+// router with split-K fp32 partials (bf16 only)
 bool proj_tc_supported(const MixParams& p);
 cudaError_t launch_proj_tc(const MixParams& p, cudaStream_t s);
+bool router_tc_supported(int B);
+int router_tc_splits(int k, int L, int Lp, int D, int B, int sms);
+cudaError_t launch_router_tc(const MixParams& p, cudaStream_t s);
 
 }  // namespace wm

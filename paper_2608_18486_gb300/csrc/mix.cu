@@ -5,13 +5,19 @@
 //   1. prenorm   : per (token, layer) inverse RMS of h_l; writes the router
 //                  input xi = [hhat_{L-1}, hhat_{L-1-p}, ...] for both branches;
 //                  per token the RoPE cos/sin at pos = slot - 1.
-//   2. router    : z = Wr[X] xi (split over the L'D reduction), fp32.
+//   2. router    : z = Wr[X] xi (split over the L'D reduction), fp32 partials;
+//                  tcgen05 for bf16 (proj_tc.cu), SIMT FMA for fp32.
 //   3. mix       : alpha = reshape(z + br), htilde_j = sum_l alpha[j][l] hhat_l,
 //                  RMSNorm_j, rounded to the projection operand dtype.
-//   4. projection: W^X_j x^X_j for every branch and channel.
-//   5. epilogue  : keys: per-head QK-norm then RoPE; keys and values are
-//                  rounded and written to the token's cache slot.
+//   4. projection: W^X_j x^X_j for every branch and channel; for bf16 on
+//                  tcgen05 with the epilogue fused (proj_tc.cu).
+//   5. epilogue  : (fp32) keys: per-head QK-norm then RoPE; keys and values
+//                  are written to the token's cache slot.
+// Every kernel is launched with programmatic dependent launch and waits for
+// its predecessor with griddepcontrol.wait before reading anything.
 #include <math.h>
+
+#include <utility>
 
 #include "common.cuh"
 #include "internal.h"
@@ -21,8 +27,61 @@ namespace wm {
 namespace {
 
 constexpr int kMixThreads = 256;
-constexpr int kMaxEPT = 16;   // D <= 4096 elements per block of 256 threads
 constexpr int kChanGroup = 4; // channels mixed per CTA
+constexpr int kVecPerThread = 2;  // 8-element vectors per thread: D <= 256*8*2
+
+__device__ __forceinline__ void pdl_wait() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                       Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, std::forward<Args>(args)...);
+}
+
+// 8 consecutive elements as fp32 (one 16-byte load for bf16, two for fp32)
+template <typename T>
+__device__ __forceinline__ void load8f(const T* src, float* f);
+template <>
+__device__ __forceinline__ void load8f<float>(const float* src, float* f) {
+  const float4 a = *reinterpret_cast<const float4*>(src);
+  const float4 c = *reinterpret_cast<const float4*>(src + 4);
+  f[0] = a.x; f[1] = a.y; f[2] = a.z; f[3] = a.w;
+  f[4] = c.x; f[5] = c.y; f[6] = c.z; f[7] = c.w;
+}
+template <>
+__device__ __forceinline__ void load8f<__nv_bfloat16>(const __nv_bfloat16* src, float* f) {
+  Elem<__nv_bfloat16>::unpack(*reinterpret_cast<const uint4*>(src), f);
+}
+template <typename T>
+__device__ __forceinline__ void store8f(T* dst, const float* f);
+template <>
+__device__ __forceinline__ void store8f<float>(float* dst, const float* f) {
+  *reinterpret_cast<float4*>(dst) = make_float4(f[0], f[1], f[2], f[3]);
+  *reinterpret_cast<float4*>(dst + 4) = make_float4(f[4], f[5], f[6], f[7]);
+}
+template <>
+__device__ __forceinline__ void store8f<__nv_bfloat16>(__nv_bfloat16* dst, const float* f) {
+  uint4 u;
+  __nv_bfloat162 t;
+  t = __floats2bfloat162_rn(f[0], f[1]); u.x = *reinterpret_cast<uint32_t*>(&t);
+  t = __floats2bfloat162_rn(f[2], f[3]); u.y = *reinterpret_cast<uint32_t*>(&t);
+  t = __floats2bfloat162_rn(f[4], f[5]); u.z = *reinterpret_cast<uint32_t*>(&t);
+  t = __floats2bfloat162_rn(f[6], f[7]); u.w = *reinterpret_cast<uint32_t*>(&t);
+  *reinterpret_cast<uint4*>(dst) = u;
+}
 
 // ---------------------------------------------------------------- prenorm
 template <typename T>
@@ -30,6 +89,7 @@ __global__ void __launch_bounds__(kMixThreads) prenorm_kernel(const MixParams p)
   __shared__ float red[32];
   __shared__ float s_r;
   const int l = blockIdx.x, b = blockIdx.y, tid = threadIdx.x;
+  pdl_wait();
   const T* hp = reinterpret_cast<const T*>(p.h) + ((int64_t)b * p.L + l) * p.D;
   float ss = 0.f;
   for (int e = tid; e < p.D; e += kMixThreads) {
@@ -49,8 +109,10 @@ __global__ void __launch_bounds__(kMixThreads) prenorm_kernel(const MixParams p)
     const int m = from_top / p.p;
     for (int X = 0; X < 2; ++X) {
       const T* g = reinterpret_cast<const T*>(p.pre_g[X]);
-      float* xo = p.xi + ((int64_t)X * p.B + b) * ((int64_t)p.Lp * p.D) + (int64_t)m * p.D;
-      for (int e = tid; e < p.D; e += kMixThreads) xo[e] = ldf(hp + e) * r * ldf(g + e);
+      T* xo = reinterpret_cast<T*>(p.xi) + ((int64_t)X * p.B + b) * ((int64_t)p.Lp * p.D) +
+              (int64_t)m * p.D;
+      for (int e = tid; e < p.D; e += kMixThreads)
+        xo[e] = Elem<T>::from_f(ldf(hp + e) * r * ldf(g + e));
     }
   }
   if (l == 0) {
@@ -110,6 +172,7 @@ __global__ void __launch_bounds__(256) gemm_wxT_simt(const GemmArgs a) {
                 (int64_t)(bi % a.per_branch) * a.w_stride;
   const TX* X = reinterpret_cast<const TX*>(a.X) + (int64_t)bi * a.x_stride;
   const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
+  pdl_wait();
   float acc[4][2] = {};
   for (int k0 = kbeg; k0 < kend; k0 += BK) {
     {  // W tile: row tid/4, 8 consecutive k
@@ -163,63 +226,105 @@ __global__ void __launch_bounds__(256) gemm_wxT_simt(const GemmArgs a) {
 }
 
 // ---------------------------------------------------------------- mix
+// One CTA per (token, branch, group of kChanGroup channels).  Thread t owns
+// the 8-element vectors t, t + 256 of D, so h, gains and the output move as
+// 16-byte vectors.
 template <typename T>
 __global__ void __launch_bounds__(kMixThreads) mix_kernel(const MixParams p) {
-  extern __shared__ float sm[];            // alpha[kChanGroup][L], r[L]
-  __shared__ float red[32];
+  extern __shared__ float sm[];  // alpha[kChanGroup][L], r[L]
+  __shared__ float red[kMixThreads / 32][kChanGroup];
   float* alpha = sm;
   float* rl = sm + kChanGroup * p.L;
   const int b = blockIdx.x, X = blockIdx.y, j0 = blockIdx.z * kChanGroup;
-  const int tid = threadIdx.x;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int nj = min(kChanGroup, p.k - j0);
   const int kL = p.k * p.L;
+  pdl_wait();
   const T* br = reinterpret_cast<const T*>(p.br[X]);
+  // alpha[j][l] = z[j*L + l] = bias + sum of the router's split partials
   for (int i = tid; i < nj * p.L; i += kMixThreads) {
-    const int o = j0 * p.L + i;  // alpha[j][l] = z[j*L + l]
+    const int o = j0 * p.L + i;
+    const float* zp = p.zpart + ((int64_t)X * p.nsplit_r * p.B + b) * kL + o;
     float z = ldf(br + o);
-    for (int s = 0; s < p.nsplit_r; ++s)
-      z += p.zpart[(((int64_t)X * p.nsplit_r + s) * p.B + b) * kL + o];
+#pragma unroll 8
+    for (int s2 = 0; s2 < p.nsplit_r; ++s2) z += zp[(int64_t)s2 * p.B * kL];
     alpha[i] = z;
   }
   for (int i = tid; i < p.L; i += kMixThreads) rl[i] = p.inv_rms[b * p.L + i];
   __syncthreads();
 
+  const int nvec = p.D / 8;
   const T* hp = reinterpret_cast<const T*>(p.h) + (int64_t)b * p.L * p.D;
   const T* g = reinterpret_cast<const T*>(p.pre_g[X]);
-  float acc[kChanGroup][kMaxEPT];
+  float gv[kVecPerThread][8];
+  float acc[kChanGroup][kVecPerThread][8];
 #pragma unroll
-  for (int jj = 0; jj < kChanGroup; ++jj)
+  for (int v = 0; v < kVecPerThread; ++v) {
+    const int vi = tid + v * kMixThreads;
+    if (vi < nvec) load8f<T>(g + vi * 8, gv[v]);
 #pragma unroll
-    for (int i = 0; i < kMaxEPT; ++i) acc[jj][i] = 0.f;
+    for (int jj = 0; jj < kChanGroup; ++jj)
+#pragma unroll
+      for (int i = 0; i < 8; ++i) acc[jj][v][i] = 0.f;
+  }
+#pragma unroll 4
   for (int l = 0; l < p.L; ++l) {
     const float r = rl[l];
+    float a[kChanGroup];
 #pragma unroll
-    for (int i = 0; i < kMaxEPT; ++i) {
-      const int e = tid + i * kMixThreads;
-      if (e < p.D) {
-        const float hv = ldf(hp + (int64_t)l * p.D + e) * r * ldf(g + e);
+    for (int jj = 0; jj < kChanGroup; ++jj) a[jj] = jj < nj ? alpha[jj * p.L + l] : 0.f;
 #pragma unroll
-        for (int jj = 0; jj < kChanGroup; ++jj)
-          if (jj < nj) acc[jj][i] = fmaf(alpha[jj * p.L + l], hv, acc[jj][i]);
+    for (int v = 0; v < kVecPerThread; ++v) {
+      const int vi = tid + v * kMixThreads;
+      if (vi < nvec) {
+        float hv[8];
+        load8f<T>(hp + (int64_t)l * p.D + vi * 8, hv);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          const float hh = hv[i] * r * gv[v][i];  // pre-mix RMSNorm with gain
+#pragma unroll
+          for (int jj = 0; jj < kChanGroup; ++jj) acc[jj][v][i] = fmaf(a[jj], hh, acc[jj][v][i]);
+        }
       }
     }
+  }
+  // per-channel sums of squares, reduced over the block for all channels at once
+  float ss[kChanGroup];
+#pragma unroll
+  for (int jj = 0; jj < kChanGroup; ++jj) {
+    float t = 0.f;
+#pragma unroll
+    for (int v = 0; v < kVecPerThread; ++v)
+#pragma unroll
+      for (int i = 0; i < 8; ++i) t = fmaf(acc[jj][v][i], acc[jj][v][i], t);
+    t = warp_sum(t);
+    if (lane == 0) red[warp][jj] = t;
+  }
+  __syncthreads();
+#pragma unroll
+  for (int jj = 0; jj < kChanGroup; ++jj) {
+    float t = 0.f;
+#pragma unroll
+    for (int w = 0; w < kMixThreads / 32; ++w) t += red[w][jj];
+    ss[jj] = rsqrtf(t / (float)p.D + p.eps_rms);
   }
   T* xop = reinterpret_cast<T*>(p.xop);
 #pragma unroll
   for (int jj = 0; jj < kChanGroup; ++jj) {
     if (jj >= nj) break;
-    float ss = 0.f;
-#pragma unroll
-    for (int i = 0; i < kMaxEPT; ++i) ss = fmaf(acc[jj][i], acc[jj][i], ss);
-    ss = block_sum(ss, red);
-    const float rr = rsqrtf(ss / (float)p.D + p.eps_rms);
     const int j = j0 + jj;
     const T* cg = reinterpret_cast<const T*>(p.ch_g[X]) + (int64_t)j * p.D;
     T* xo = xop + (((int64_t)X * p.k + j) * p.B + b) * p.D;
 #pragma unroll
-    for (int i = 0; i < kMaxEPT; ++i) {
-      const int e = tid + i * kMixThreads;
-      if (e < p.D) xo[e] = Elem<T>::from_f(acc[jj][i] * rr * ldf(cg + e));
+    for (int v = 0; v < kVecPerThread; ++v) {
+      const int vi = tid + v * kMixThreads;
+      if (vi < nvec) {
+        float cv[8], o[8];
+        load8f<T>(cg + vi * 8, cv);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) o[i] = acc[jj][v][i] * ss[jj] * cv[i];
+        store8f<T>(xo + vi * 8, o);
+      }
     }
   }
 }
@@ -230,6 +335,7 @@ __global__ void __launch_bounds__(128) kv_epilogue_kernel(const MixParams p) {
   constexpr int EPL = HD / 32;  // elements per lane; pairs (e, e + HD/2) share a lane
   const int b = blockIdx.x, j = blockIdx.y, X = blockIdx.z;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  pdl_wait();
   const int s = p.slot[b];
   if (s < 1 || s >= p.max_pages * p.P) {
     if (threadIdx.x == 0 && j == 0 && X == 0) report(p.status, WM_ERR_BOUNDS);
@@ -277,8 +383,12 @@ __global__ void __launch_bounds__(128) kv_epilogue_kernel(const MixParams p) {
 template <typename T>
 cudaError_t launch_all(MixParams& p, cudaStream_t s) {
   const int kL = p.k * p.L;
-  prenorm_kernel<T><<<dim3(p.L, p.B), kMixThreads, 0, s>>>(p);
-  {
+  const bool bf16 = sizeof(T) == 2;
+  cudaError_t e = launch_pdl(prenorm_kernel<T>, dim3(p.L, p.B), dim3(kMixThreads), 0, s, p);
+  if (e != cudaSuccess) return e;
+  if (bf16 && router_tc_supported(p.B)) {
+    e = launch_router_tc(p, s);
+  } else {
     GemmArgs a{};
     a.W[0] = p.Wr[0];
     a.W[1] = p.Wr[1];
@@ -293,17 +403,17 @@ cudaError_t launch_all(MixParams& p, cudaStream_t s) {
     a.nsplit = p.nsplit_r;
     a.k_per_split = ((a.K + p.nsplit_r - 1) / p.nsplit_r + BK - 1) / BK * BK;
     dim3 grid((a.M + BM - 1) / BM, (a.N + BN - 1) / BN, 2 * a.nsplit);
-    gemm_wxT_simt<T, float><<<grid, 256, 0, s>>>(a);
+    e = launch_pdl(gemm_wxT_simt<T, T>, grid, dim3(256), 0, s, a);
   }
+  if (e != cudaSuccess) return e;
   {
     const size_t smem = sizeof(float) * (kChanGroup * p.L + p.L);
     dim3 grid(p.B, 2, (p.k + kChanGroup - 1) / kChanGroup);
-    mix_kernel<T><<<grid, kMixThreads, smem, s>>>(p);
-  }
-  if (sizeof(T) == 2 && proj_tc_supported(p)) {
-    // bf16: tensor-core projection, QK-norm, RoPE and cache write in one kernel
-    cudaError_t e = cudaGetLastError();
+    e = launch_pdl(mix_kernel<T>, grid, dim3(kMixThreads), smem, s, p);
     if (e != cudaSuccess) return e;
+  }
+  if (bf16 && proj_tc_supported(p)) {
+    // bf16: tensor-core projection, QK-norm, RoPE and cache write in one kernel
     return launch_proj_tc(p, s);
   }
   {
@@ -321,16 +431,14 @@ cudaError_t launch_all(MixParams& p, cudaStream_t s) {
     a.nsplit = 1;
     a.k_per_split = p.D;
     dim3 grid((a.M + BM - 1) / BM, (a.N + BN - 1) / BN, 2 * p.k);
-    gemm_wxT_simt<T, T><<<grid, 256, 0, s>>>(a);
+    e = launch_pdl(gemm_wxT_simt<T, T>, grid, dim3(256), 0, s, a);
+    if (e != cudaSuccess) return e;
   }
   {
     dim3 grid(p.B, p.k, 2);
-    if (p.d == 64)
-      kv_epilogue_kernel<T, 64><<<grid, 128, 0, s>>>(p);
-    else
-      kv_epilogue_kernel<T, 128><<<grid, 128, 0, s>>>(p);
+    if (p.d == 64) return launch_pdl(kv_epilogue_kernel<T, 64>, grid, dim3(128), 0, s, p);
+    return launch_pdl(kv_epilogue_kernel<T, 128>, grid, dim3(128), 0, s, p);
   }
-  return cudaGetLastError();
 }
 
 size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
@@ -342,18 +450,23 @@ MixWorkspace mix_workspace_layout(const wm_config& cfg, int32_t B, int sm_count)
   const int Lp = (cfg.L + cfg.p - 1) / cfg.p;
   const int kL = cfg.k * cfg.L;
   const int64_t Kr = (int64_t)Lp * cfg.D;
-  const int tiles = 2 * ((kL + BM - 1) / BM) * ((B + BN - 1) / BN);
-  int ns = (2 * sm_count + tiles - 1) / tiles;
-  const int max_split = (int)((Kr + 255) / 256);
-  ns = ns < 1 ? 1 : (ns > max_split ? max_split : ns);
-  // same rounding as the launch: whole BK blocks per split
-  const int64_t kps = ((Kr + ns - 1) / ns + BK - 1) / BK * BK;
-  ns = (int)((Kr + kps - 1) / kps);
+  int ns;
+  if (cfg.dtype == WM_DT_BF16 && router_tc_supported(B)) {
+    ns = router_tc_splits(cfg.k, cfg.L, Lp, cfg.D, B, sm_count);
+  } else {
+    const int tiles = 2 * ((kL + BM - 1) / BM) * ((B + BN - 1) / BN);
+    ns = (2 * sm_count + tiles - 1) / tiles;
+    const int max_split = (int)((Kr + 255) / 256);
+    ns = ns < 1 ? 1 : (ns > max_split ? max_split : ns);
+    // same rounding as the launch: whole BK blocks per split
+    const int64_t kps = ((Kr + ns - 1) / ns + BK - 1) / BK * BK;
+    ns = (int)((Kr + kps - 1) / kps);
+  }
   w.nsplit_r = ns;
   const size_t esz = cfg.dtype == WM_DT_F32 ? 4 : 2;
   size_t off = 0;
   w.inv_rms = off; off += align256(sizeof(float) * B * cfg.L);
-  w.xi = off;      off += align256(sizeof(float) * 2 * (size_t)B * Kr);
+  w.xi = off;      off += align256(esz * 2 * (size_t)B * Kr);
   w.zpart = off;   off += align256(sizeof(float) * 2 * (size_t)ns * B * kL);
   w.rope_cs = off; off += align256(sizeof(float) * (size_t)B * cfg.d);
   w.xop = off;     off += align256(esz * 2 * (size_t)cfg.k * B * cfg.D);

@@ -1,7 +1,11 @@
-// Per-channel K/V projection on the tcgen05 tensor cores with a fused
-// epilogue (Sec. 3.1 Step 2): K_j = W^K_j x^K_j, V_j = W^V_j x^V_j for the
-// B tokens of a decode step, then per-head QK-norm and RoPE on keys, bf16
-// rounding and the write to each token's cache slot.
+// The two dense contractions of the cross-layer KV pool on the tcgen05
+// tensor cores (bf16 operands, fp32 accumulation in TMEM):
+//  * the per-channel K/V projection with a fused epilogue (Sec. 3.1 Step 2):
+//    K_j = W^K_j x^K_j, V_j = W^V_j x^V_j for the B tokens of a decode step,
+//    then per-head QK-norm and RoPE on keys, bf16 rounding and the write to
+//    each token's cache slot;
+//  * the router logits W^alpha xi (Sec. 3.1 Step 1), split over the long L'D
+//    reduction, each split storing fp32 partial sums.
 //
 // Shape: at decode the token count B is small (16..64) while the weights
 // are large (Hkv*d x D per channel and branch), so the weights take the MMA's
@@ -24,11 +28,17 @@ namespace {
 
 constexpr int kTcM = 128;      // weight rows per tile (MMA M)
 constexpr int kTcBK = 64;      // K elements per stage (128 bytes of bf16)
-constexpr int kTcStages = 4;
+constexpr int kTcMaxStages = 12;
 constexpr int kTcThreads = 128;
+constexpr int kTcMaxTokens = 256;
+
+enum { kEpiKV = 0, kEpiPartial = 1 };
 
 struct ProjTcParams {
-  int32_t k, B, Hkv, D, M_item, BN, nk;
+  int32_t k, B, Hkv, D, M_item, BN, nk, stages;
+  int32_t kb_per_split, M_total;  // router: k-blocks per split, rows of W
+  int32_t rope_smem_off;          // projection: byte offset of the RoPE table in smem, 0 = global
+  float* zpart;                   // router: [2][nsplit][B][M_total]
   int32_t P, log2P, num_pages, max_pages;
   uint32_t tmem_cols;
   float eps_qk;
@@ -41,16 +51,20 @@ struct ProjTcParams {
   int32_t* status;
 };
 
-template <int HD>
+// MODE kEpiKV: grid (Hkv*d/128, k, 2) = (row tile, channel j, branch X).
+// MODE kEpiPartial: grid (ceil(kL/128), nsplit, 2) = (row tile, split, branch X).
+template <int HD, int MODE>
 __global__ void __launch_bounds__(kTcThreads, 1)
     proj_tc_kernel(const __grid_constant__ CUtensorMap tmW0, const __grid_constant__ CUtensorMap tmW1,
                    const __grid_constant__ CUtensorMap tmX, const ProjTcParams p) {
   constexpr int EPL = HD / 32;
   extern __shared__ uint8_t smem_dyn[];
-  __shared__ uint64_t full[kTcStages], empty[kTcStages], done;
+  __shared__ uint64_t full[kTcMaxStages], empty[kTcMaxStages], done;
   __shared__ uint32_t tmem_base;
+  __shared__ int s_slot[kTcMaxTokens], s_page[kTcMaxTokens];
 
   const int mt = blockIdx.x, j = blockIdx.y, X = blockIdx.z;
+  const int NS = p.stages;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const CUtensorMap* tmW = X == 0 ? &tmW0 : &tmW1;
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_dyn) + 1023) &
@@ -58,10 +72,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   const uint32_t a_bytes = kTcM * 128;
   const uint32_t b_bytes = (uint32_t)p.BN * 128;
   uint8_t* As = base;
-  uint8_t* Bs = base + kTcStages * a_bytes;
+  uint8_t* Bs = base + NS * a_bytes;
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kTcStages; ++s) {
+    for (int s = 0; s < NS; ++s) {
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
     }
@@ -69,6 +83,22 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     fence_mbar_init();
     tc::prefetch_tensormap(tmW);
     tc::prefetch_tensormap(&tmX);
+  }
+  // programmatic dependent launch: inputs may come from the previous grid
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  float* rope_s = reinterpret_cast<float*>(base + p.rope_smem_off);  // [B][HD/2][2] or unused
+  if (MODE == kEpiKV) {
+    if (p.rope_smem_off > 0)
+      for (int i = threadIdx.x; i < p.B * HD; i += kTcThreads) rope_s[i] = p.rope_cs[i];
+    // destination slot and page of every token, read before the K loop
+    for (int n = threadIdx.x; n < p.B; n += kTcThreads) {
+      const int s = p.slot[n];
+      int pg = -1;
+      if (s >= 1 && s < p.max_pages * p.P) pg = p.page_table[(int64_t)n * p.max_pages + (s >> p.log2P)];
+      s_slot[n] = s;
+      s_page[n] = (pg >= 0 && pg < p.num_pages) ? pg : -1;
+    }
   }
   if (warp == 0) {
     tc::tmem_alloc(&tmem_base, p.tmem_cols);
@@ -78,27 +108,30 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   __syncthreads();
   tc::fence_after_sync();
   const uint32_t tmem = tmem_base;
-  const int wrow = j * p.M_item + mt * kTcM;
-  const int xrow = (X * p.k + j) * p.B;
+  const int wrow = MODE == kEpiKV ? j * p.M_item + mt * kTcM : mt * kTcM;
+  const int xrow = MODE == kEpiKV ? (X * p.k + j) * p.B : X * p.B;
+  const int kb0 = MODE == kEpiKV ? 0 : j * p.kb_per_split;
+  const int kb1 = MODE == kEpiKV ? p.nk : min(p.nk, kb0 + p.kb_per_split);
+  const int nkb = kb1 - kb0;
 
   if (warp == 0 && lane == 0) {
     // TMA producer
-    for (int kb = 0; kb < p.nk; ++kb) {
-      const int s = kb % kTcStages;
-      if (kb >= kTcStages && !mbar_wait(&empty[s], ((kb / kTcStages) - 1) & 1)) {
+    for (int kb = 0; kb < nkb; ++kb) {
+      const int s = kb % NS;
+      if (kb >= NS && !mbar_wait(&empty[s], ((kb / NS) - 1) & 1)) {
         report(p.status, WM_ERR_TIMEOUT);
         break;
       }
       mbar_arrive_expect_tx(&full[s], a_bytes + b_bytes);
-      tc::tma_load_2d(As + s * a_bytes, tmW, kb * kTcBK, wrow, &full[s]);
-      tc::tma_load_2d(Bs + s * b_bytes, &tmX, kb * kTcBK, xrow, &full[s]);
+      tc::tma_load_2d(As + s * a_bytes, tmW, (kb0 + kb) * kTcBK, wrow, &full[s]);
+      tc::tma_load_2d(Bs + s * b_bytes, &tmX, (kb0 + kb) * kTcBK, xrow, &full[s]);
     }
   } else if (warp == 1 && lane == 0) {
     // MMA issuer: 4 MMAs of K = 16 per stage
     const uint32_t idesc = tc::idesc_bf16_f32(kTcM, p.BN);
-    for (int kb = 0; kb < p.nk; ++kb) {
-      const int s = kb % kTcStages;
-      if (!mbar_wait(&full[s], (kb / kTcStages) & 1)) {
+    for (int kb = 0; kb < nkb; ++kb) {
+      const int s = kb % NS;
+      if (!mbar_wait(&full[s], (kb / NS) & 1)) {
         report(p.status, WM_ERR_TIMEOUT);
         break;
       }
@@ -139,22 +172,30 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   }
   if (!ok) return;
 
+  if (MODE == kEpiPartial) {
+    // fp32 partial logits of this split: zpart[X][split][n][row]
+    float* z = p.zpart + (((int64_t)X * gridDim.y + j) * p.B) * p.M_total;
+    const int m0 = mt * kTcM;
+    for (int i = threadIdx.x; i < p.B * kTcM; i += kTcThreads) {
+      const int n = i / kTcM, r = i % kTcM;
+      if (m0 + r < p.M_total) z[(int64_t)n * p.M_total + m0 + r] = T[n * kTcM + r];
+    }
+    return;
+  }
   // per (token, head) epilogue: keys QK-norm + RoPE, bf16 write to the cache slot
   const int hpt = kTcM / HD;
   const bool reporter = (mt == 0 && j == 0 && X == 0);
   __nv_bfloat16* pool = X == 0 ? p.k_pool : p.v_pool;
-  const __nv_bfloat16* qg = p.qk_g + (int64_t)j * HD;
+  float qgv[EPL];  // QK-norm gain of channel j, the same for every item of this CTA
+#pragma unroll
+  for (int i = 0; i < EPL; ++i) qgv[i] = __bfloat162float(p.qk_g[(int64_t)j * HD + lane + 32 * i]);
+  const float* cs_tab = p.rope_smem_off > 0 ? rope_s : p.rope_cs;
   for (int it = warp; it < p.B * hpt; it += kTcThreads / 32) {
     const int n = it / hpt, hl = it % hpt;
     const int hh = mt * hpt + hl;
-    const int s = p.slot[n];
-    if (s < 1 || s >= p.max_pages * p.P) {
-      if (reporter && lane == 0) report(p.status, WM_ERR_BOUNDS);
-      continue;
-    }
-    const int pg = p.page_table[(int64_t)n * p.max_pages + (s >> p.log2P)];
-    if (pg < 0 || pg >= p.num_pages) {
-      if (reporter && lane == 0) report(p.status, WM_ERR_BOUNDS);
+    const int s = s_slot[n], pg = s_page[n];
+    if (pg < 0) {
+      if (reporter && hl == 0 && lane == 0) report(p.status, WM_ERR_BOUNDS);
       continue;
     }
     float y[EPL];
@@ -167,12 +208,12 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       ss = warp_sum(ss);
       const float rr = rsqrtf(ss / (float)HD + p.eps_qk);
 #pragma unroll
-      for (int i = 0; i < EPL; ++i) y[i] = y[i] * rr * __bfloat162float(qg[lane + 32 * i]);
+      for (int i = 0; i < EPL; ++i) y[i] = y[i] * rr * qgv[i];
 #pragma unroll
       for (int i = 0; i < EPL / 2; ++i) {
         const int e = lane + 32 * i;
-        const float cs = p.rope_cs[((int64_t)n * (HD / 2) + e) * 2];
-        const float sn = p.rope_cs[((int64_t)n * (HD / 2) + e) * 2 + 1];
+        const float2 csn = reinterpret_cast<const float2*>(cs_tab)[n * (HD / 2) + e];
+        const float cs = csn.x, sn = csn.y;
         const float x0 = y[i], x1 = y[i + EPL / 2];
         y[i] = x0 * cs - x1 * sn;
         y[i + EPL / 2] = x1 * cs + x0 * sn;
@@ -217,10 +258,70 @@ uint32_t pow2_at_least(uint32_t x, uint32_t lo) {
   return r;
 }
 
+int sm_count_cur() {
+  int dev = 0, n = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
+    n = 148;
+  return n;
+}
+
+// Pipeline depth: deep enough to keep one round trip of weights in flight;
+// shallow enough for two CTAs per SM when the grid has more than one wave.
+int pick_stages(int nkb, int BN, int64_t grid, int sms) {
+  const int stage_bytes = kTcM * 128 + BN * 128;
+  const int budget = grid > sms ? 100 * 1024 : 200 * 1024;
+  int ns = budget / stage_bytes;
+  ns = ns < 2 ? 2 : (ns > kTcMaxStages ? kTcMaxStages : ns);
+  return ns > nkb ? (nkb < 2 ? 2 : nkb) : ns;
+}
+
+size_t tc_smem(int stages, int BN) {
+  const size_t pipe = (size_t)stages * (kTcM * 128 + BN * 128);
+  const size_t tile = (size_t)BN * kTcM * sizeof(float);  // epilogue reuses the stages
+  return (pipe > tile ? pipe : tile) + 1024;
+}
+
+template <int HD, int MODE>
+cudaError_t launch_mode(dim3 grid, size_t smem, const CUtensorMap& w0, const CUtensorMap& w1,
+                        const CUtensorMap& x, const ProjTcParams& p, cudaStream_t s) {
+  static size_t smem_set = 0;
+  auto kern = proj_tc_kernel<HD, MODE>;
+  if (smem > smem_set) {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    smem_set = smem;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = dim3(kTcThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, w0, w1, x, p);
+}
+
 }  // namespace
 
 bool proj_tc_supported(const MixParams& mp) {
-  return (mp.Hkv * mp.d) % kTcM == 0 && mp.B >= 1 && mp.B <= 256 && encode_fn() != nullptr;
+  return (mp.Hkv * mp.d) % kTcM == 0 && mp.B >= 1 && mp.B <= kTcMaxTokens && encode_fn() != nullptr;
+}
+
+bool router_tc_supported(int B) { return B >= 1 && B <= kTcMaxTokens; }
+
+int router_tc_splits(int k, int L, int Lp, int D, int B, int sms) {
+  const int nk = (Lp * D + kTcBK - 1) / kTcBK;
+  const int tiles = 2 * ((k * L + kTcM - 1) / kTcM);
+  int ns = (sms + tiles - 1) / tiles;
+  const int max_ns = nk / 8 > 1 ? nk / 8 : 1;  // at least 8 k-blocks per split
+  ns = ns < 1 ? 1 : (ns > max_ns ? max_ns : ns);
+  const int per = (nk + ns - 1) / ns;
+  (void)B;
+  return (nk + per - 1) / per;
 }
 
 cudaError_t launch_proj_tc(const MixParams& mp, cudaStream_t s) {
@@ -251,19 +352,41 @@ cudaError_t launch_proj_tc(const MixParams& mp, cudaStream_t s) {
       return cudaErrorInvalidValue;
   if (!encode_kmajor(&tmX, mp.xop, (uint64_t)2 * mp.k * mp.B, mp.D, (uint32_t)p.BN))
     return cudaErrorInvalidValue;
-  const size_t smem = (size_t)kTcStages * (kTcM * 128 + p.BN * 128) + 1024;
   dim3 grid(p.M_item / kTcM, mp.k, 2);
-  cudaError_t e;
-  if (mp.d == 64) {
-    e = cudaFuncSetAttribute(proj_tc_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    proj_tc_kernel<64><<<grid, kTcThreads, smem, s>>>(tmW[0], tmW[1], tmX, p);
-  } else {
-    e = cudaFuncSetAttribute(proj_tc_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    proj_tc_kernel<128><<<grid, kTcThreads, smem, s>>>(tmW[0], tmW[1], tmX, p);
+  p.stages = pick_stages(p.nk, p.BN, (int64_t)grid.x * grid.y * grid.z, sm_count_cur());
+  size_t smem = tc_smem(p.stages, p.BN);
+  const size_t rope_bytes = (size_t)mp.B * mp.d * sizeof(float);
+  if (smem + rope_bytes <= 200 * 1024) {
+    p.rope_smem_off = (int32_t)(smem - 1024);  // offset from the 1 KB-aligned base
+    smem += rope_bytes;
   }
-  return cudaGetLastError();
+  if (mp.d == 64) return launch_mode<64, kEpiKV>(grid, smem, tmW[0], tmW[1], tmX, p, s);
+  return launch_mode<128, kEpiKV>(grid, smem, tmW[0], tmW[1], tmX, p, s);
+}
+
+cudaError_t launch_router_tc(const MixParams& mp, cudaStream_t s) {
+  ProjTcParams p{};
+  const int kL = mp.k * mp.L;
+  const int K = mp.Lp * mp.D;
+  p.k = mp.k;
+  p.B = mp.B;
+  p.D = K;
+  p.BN = (mp.B + 15) / 16 * 16;
+  p.nk = (K + kTcBK - 1) / kTcBK;
+  p.kb_per_split = (p.nk + mp.nsplit_r - 1) / mp.nsplit_r;
+  p.M_total = kL;
+  p.zpart = mp.zpart;
+  p.tmem_cols = pow2_at_least((uint32_t)p.BN, 32);
+  p.status = mp.status;
+  CUtensorMap tmW[2], tmX;
+  for (int X = 0; X < 2; ++X)
+    if (!encode_kmajor(&tmW[X], mp.Wr[X], (uint64_t)kL, K, kTcM)) return cudaErrorInvalidValue;
+  if (!encode_kmajor(&tmX, mp.xi, (uint64_t)2 * mp.B, K, (uint32_t)p.BN))
+    return cudaErrorInvalidValue;
+  dim3 grid((kL + kTcM - 1) / kTcM, mp.nsplit_r, 2);
+  p.stages = pick_stages(p.kb_per_split, p.BN, (int64_t)grid.x * grid.y * grid.z, sm_count_cur());
+  const size_t smem = tc_smem(p.stages, p.BN);
+  return launch_mode<64, kEpiPartial>(grid, smem, tmW[0], tmW[1], tmX, p, s);
 }
 
 }  // namespace wm

@@ -36,7 +36,7 @@ bool aligned(const void* p, size_t a) { return ((uintptr_t)p % a) == 0; }
 
 // Persistent grid of one attention launch and its workspace layout.
 struct AttnPlan {
-  int stage_bytes, grid, nwarps;
+  int stage_bytes, grid, nwarps, chunk_stages, max_chunks;
   size_t off_part_o, off_part_ml, off_counters, total;
 };
 
@@ -45,6 +45,14 @@ constexpr int kAttnMaxBatch = 4096;
 // table width) use 4 KB stages and 4 CTAs per SM (16 warps: more latency
 // hiding for short launches); larger ones use 8 KB stages and 2 CTAs per SM.
 constexpr double kAttnSmallLaunchBytes = 1.0e9;
+// Launches reading at least this many KV bytes hand out work dynamically:
+// chunks of the stage stream taken from an atomic counter, about
+// kAttnChunksPerWarp per warp, so warps that stream faster take more.
+// Smaller launches split statically, one chunk per warp: their chunk ends
+// (partial publish + ticket) would cost more than the balance gains.
+constexpr double kAttnDynamicLaunchBytes = 2.0e9;
+constexpr int kAttnChunksPerWarp = 8;
+constexpr int kAttnMinChunkStages = 4;  // > the per-warp ring depth
 
 AttnPlan attn_plan(const wm_config& c, int32_t B, int32_t max_pages) {
   AttnPlan pl{};
@@ -62,14 +70,24 @@ AttnPlan attn_plan(const wm_config& c, int32_t B, int32_t max_pages) {
   if (grid < 1) grid = 1;
   pl.grid = (int)grid;
   pl.nwarps = (int)grid * wpc;
+  if (kv_bytes >= kAttnDynamicLaunchBytes) {
+    int64_t ch = (ns_max + (int64_t)pl.nwarps * kAttnChunksPerWarp - 1) /
+                 ((int64_t)pl.nwarps * kAttnChunksPerWarp);
+    if (ch < kAttnMinChunkStages) ch = kAttnMinChunkStages;
+    pl.chunk_stages = (int)ch;
+    pl.max_chunks = (int)(ns_max / ch > 1 ? ns_max / ch : 1);  // the remainder joins the last chunk
+  } else {
+    pl.chunk_stages = 0;        // static: the kernel sizes one chunk per warp
+    pl.max_chunks = pl.nwarps;  // at most one chunk per warp
+  }
   const int G = c.Hq / c.Hkv;
   size_t off = 0;
   pl.off_part_o = off;
-  off += align256(sizeof(float) * 2 * (size_t)pl.nwarps * G * c.d);
+  off += align256(sizeof(float) * 2 * (size_t)pl.max_chunks * G * c.d);
   pl.off_part_ml = off;
-  off += align256(sizeof(float) * 2 * (size_t)pl.nwarps * G * 2);
+  off += align256(sizeof(float) * 2 * (size_t)pl.max_chunks * G * 2);
   pl.off_counters = off;
-  off += align256(sizeof(int32_t) * (size_t)B * c.Hkv);
+  off += align256(sizeof(int32_t) * ((size_t)B * c.Hkv + 1));
   pl.total = off;
   return pl;
 }
@@ -186,7 +204,8 @@ wm_status wm_decode_attn(const wm_config* c, const wm_cache* cache, int32_t laye
   p.num_pages = cache->num_pages;
   p.max_pages = max_pages;
   p.B = B;
-  p.nwarps = pl.nwarps;
+  p.chunk_stages = pl.chunk_stages;
+  p.max_chunks = pl.max_chunks;
   p.qscale = (float)(1.4426950408889634 / sqrt((double)c->d));
   cudaError_t e = wm::launch_decode_attn(p, pl.stage_bytes, c->dtype, c->d, c->Hq / c->Hkv,
                                          pl.grid, (cudaStream_t)stream);
@@ -250,7 +269,7 @@ wm_status wm_kv_mix(const wm_config* c, const wm_cache* cache, const wm_mix_weig
   p.v_pool = cache->v_pool;
   char* base = (char*)workspace;
   p.inv_rms = (float*)(base + ws.inv_rms);
-  p.xi = (float*)(base + ws.xi);
+  p.xi = base + ws.xi;
   p.zpart = (float*)(base + ws.zpart);
   p.rope_cs = (float*)(base + ws.rope_cs);
   p.xop = base + ws.xop;

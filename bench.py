@@ -263,8 +263,9 @@ def run_gpu(args, w):
         if ev_attn is not None:
             ev_attn[0].record(stream)
         for layer in range(w.L):
+            # layers after the first read nothing the previous launch wrote but q
             sess.decode_attn(layer, dp.q[layer], dp.page_table, dp.seq_lens, outs[layer],
-                             stream=stream)
+                             stream=stream, inputs_ready=layer > 0)
         if ev_attn is not None:
             ev_attn[1].record(stream)
         sess.kv_mix(dp.h, dp.page_table, dp.slot, stream=stream)

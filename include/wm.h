@@ -181,6 +181,29 @@ wm_status wm_decode_attn(const wm_config* cfg, const wm_cache* cache, int32_t la
                          int32_t B, int32_t max_pages, void* out, void* workspace,
                          size_t ws_bytes, int32_t* dev_status, void* stream);
 
+/* Flags of wm_decode_attn_flags. */
+#define WM_ATTN_INPUTS_READY 1u
+
+/*
+ * wm_decode_attn with flags; wm_decode_attn(...) is wm_decode_attn_flags(...,
+ * flags = 0, ...).  Launches are chained with programmatic dependent launch:
+ * a launch may start while the previous work on the stream finishes, and
+ * waits for it before reading anything that work may have written.
+ *   WM_ATTN_INPUTS_READY: the caller promises that the work immediately
+ *     before this call on `stream` writes none of the cache pools, the page
+ *     table, seq_lens and the workspace (it may write q).  The kernel then
+ *     starts fetching K/V while that work finishes and waits for it only
+ *     before reading q.  Within one decode step this holds for layers
+ *     1..L-1; it does NOT hold for the first layer after wm_kv_mix or after
+ *     any update of seq_lens / the page table.
+ * Unknown flag bits return WM_ERR_INVALID_ARG.
+ */
+wm_status wm_decode_attn_flags(const wm_config* cfg, const wm_cache* cache, int32_t layer,
+                               const void* q, const int32_t* page_table,
+                               const int32_t* seq_lens, int32_t B, int32_t max_pages, void* out,
+                               void* workspace, size_t ws_bytes, uint32_t flags,
+                               int32_t* dev_status, void* stream);
+
 /*
  * Decode attention for callers that cannot allocate device memory.
  *

@@ -17,7 +17,9 @@ WM_OK, WM_ERR_INVALID_ARG, WM_ERR_UNSUPPORTED, WM_ERR_CUDA, WM_ERR_BOUNDS, WM_ER
 WM_DT_F32, WM_DT_BF16 = 0, 1
 
 EXPORTED = ["wm_status_string", "wm_config_check", "wm_cache_bytes", "wm_cache_alloc",
-            "wm_kv_mix_workspace", "wm_kv_mix", "wm_decode_attn_workspace", "wm_decode_attn"]
+            "wm_kv_mix_workspace", "wm_kv_mix", "wm_decode_attn_workspace", "wm_decode_attn",
+            "wm_decode_attn_flags"]
+WM_ATTN_INPUTS_READY = 1
 
 
 class wm_config(ctypes.Structure):
@@ -76,6 +78,9 @@ def lib():
         L.wm_decode_attn.restype = ctypes.c_int
         L.wm_decode_attn.argtypes = [cp, ctypes.POINTER(wm_cache), i32, vp, vp, vp, i32, i32, vp,
                                      vp, sz, vp, vp]
+        L.wm_decode_attn_flags.restype = ctypes.c_int
+        L.wm_decode_attn_flags.argtypes = [cp, ctypes.POINTER(wm_cache), i32, vp, vp, vp, i32, i32,
+                                           vp, vp, sz, ctypes.c_uint32, vp, vp]
         _lib = L
     return _lib
 
@@ -153,6 +158,14 @@ def wm_decode_attn(cfg, cache, layer, q, page_table, seq_lens, B, max_pages, out
     return lib().wm_decode_attn(ctypes.byref(cfg), ctypes.byref(cache), int(layer), _p(q),
                                 _p(page_table), _p(seq_lens), int(B), int(max_pages), _p(out),
                                 _p(workspace), int(ws_bytes), _p(dev_status), stream)
+
+
+def wm_decode_attn_flags(cfg, cache, layer, q, page_table, seq_lens, B, max_pages, out, workspace,
+                         ws_bytes, flags, dev_status, stream) -> int:
+    return lib().wm_decode_attn_flags(ctypes.byref(cfg), ctypes.byref(cache), int(layer), _p(q),
+                                      _p(page_table), _p(seq_lens), int(B), int(max_pages),
+                                      _p(out), _p(workspace), int(ws_bytes), int(flags),
+                                      _p(dev_status), stream)
 
 
 def wm_decode_attn_noalloc(cfg, cache, layer, q, page_table, seq_lens, B, max_pages, out,

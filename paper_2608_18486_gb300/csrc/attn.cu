@@ -215,6 +215,7 @@ __global__ void __launch_bounds__(kThreads, SB == 4096 ? 4 : 2) decode_attn_kern
   int* pre = reinterpret_cast<int*>(qring + kWarps * kWStages * G * HD);  // [B+1]
   int* lens = pre + p.B + 1;                                      // [B]
   __shared__ uint64_t bars[kWarps][kWStages];
+  __shared__ uint64_t qbars[kWarps];  // query of the warp's first piece
   __shared__ uint64_t masks[kWarps][kWStages];
   __shared__ int scan[kThreads];
 
@@ -223,10 +224,14 @@ __global__ void __launch_bounds__(kThreads, SB == 4096 ? 4 : 2) decode_attn_kern
   const int max_slots = p.max_pages * p.P;
 
   // Programmatic dependent launch: the next grid on the stream may be
-  // scheduled now (it waits for this one before reading anything), and this
-  // grid waits here until the previous one has finished and flushed.
+  // scheduled now.  This grid waits for the previous one (finished and
+  // flushed) before reading anything it may have written.  With the caller's
+  // promise that the previous grid wrote neither the cache, the page table,
+  // the lengths nor the workspace (inputs_ready), the wait moves down to just
+  // before the query is read, and the first K/V copies overlap its tail.
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-  asm volatile("griddepcontrol.wait;" ::: "memory");
+  const bool early = p.inputs_ready != 0;
+  if (!early) asm volatile("griddepcontrol.wait;" ::: "memory");
 
   // ---- stages per sequence and their prefix sums (every CTA, all threads)
   {
@@ -253,13 +258,16 @@ __global__ void __launch_bounds__(kThreads, SB == 4096 ? 4 : 2) decode_attn_kern
       run += lens[i] ? (lens[i] + STAGE_SLOTS - 1) / STAGE_SLOTS : 0;
     }
     if (tid == kThreads - 1) pre[B] = scan[tid];
-    if (lane == 0)
+    if (lane == 0) {
       for (int s = 0; s < kWStages; ++s) mbar_init(&bars[warp][s], 1);
+      mbar_init(&qbars[warp], 1);
+    }
     fence_mbar_init();
     __syncthreads();
   }
   // ---- sequences with an invalid length: zero output rows, report once
   if (blockIdx.x == 0) {
+    if (early) asm volatile("griddepcontrol.wait;" ::: "memory");
     for (int b = 0; b < B; ++b) {
       if (lens[b] != 0) continue;
       T* o = reinterpret_cast<T*>(p.out) + (int64_t)b * p.Hq * HD;
@@ -297,6 +305,7 @@ __global__ void __launch_bounds__(kThreads, SB == 4096 ? 4 : 2) decode_attn_kern
     return GW + __shfl_sync(FULLMASK, grab_t, 0);
   };
   if (gw >= nchunks || NS == 0) {
+    if (early) asm volatile("griddepcontrol.wait;" ::: "memory");
     grab_issue();
     grab_take();
     return;  // warp-level from here on: no block barriers below
@@ -333,7 +342,6 @@ __global__ void __launch_bounds__(kThreads, SB == 4096 ? 4 : 2) decode_attn_kern
 
   // ---- producer: walks its chunks stage by stage, kWStages ahead of the consumer
   int64_t p_chunk = gw;
-  grab_issue();                                 // the next chunk, requested one ahead
   int64_t px = chunk_begin(p_chunk), pend = chunk_end_x(p_chunk);
   int64_t chunk_for_consumer = -1;              // the producer's chunk after a switch
   bool p_done = false;
@@ -349,7 +357,9 @@ __global__ void __launch_bounds__(kThreads, SB == 4096 ? 4 : 2) decode_attn_kern
     T* kd = myring + buf * 2 * STAGE_ELEMS;
     T* vd = kd + STAGE_ELEMS;
     uint64_t* bar = &bars[warp][buf];
-    const uint32_t qb = first ? Q_BYTES : 0u;
+    // the first piece's query arrives on qbars (issued after the dependency wait)
+    const bool with_q = first && pseq > 0;
+    const uint32_t qb = with_q ? Q_BYTES : 0u;
     const T* qsrc = reinterpret_cast<const T*>(p.q) + ((int64_t)pc.b * p.Hq + pc.h * G) * HD;
     if (p.P >= STAGE_SLOTS) {
       const int pg = page_of(pc.b, s_begin >> p.log2P, 0);
@@ -363,7 +373,7 @@ __global__ void __launch_bounds__(kThreads, SB == 4096 ? 4 : 2) decode_attn_kern
           bulk_g2s(kd, kb + off, KV_BYTES, bar, policy);
           bulk_g2s(vd, vb + off, KV_BYTES, bar, policy);
         }
-        if (first) bulk_g2s(myq + buf * G * HD, qsrc, Q_BYTES, bar, policy);
+        if (with_q) bulk_g2s(myq + buf * G * HD, qsrc, Q_BYTES, bar, policy);
       }
     } else {
       const int npp = STAGE_SLOTS >> p.log2P;  // pages per stage (<= 32)
@@ -377,7 +387,7 @@ __global__ void __launch_bounds__(kThreads, SB == 4096 ? 4 : 2) decode_attn_kern
         masks[warp][buf] = mask;
         if (__popc(mask) < lpn) report(p.status, WM_ERR_BOUNDS);
         mbar_arrive_expect_tx(bar, 2u * bytes * (uint32_t)__popc(mask) + qb);
-        if (first) bulk_g2s(myq + buf * G * HD, qsrc, Q_BYTES, bar, policy);
+        if (with_q) bulk_g2s(myq + buf * G * HD, qsrc, Q_BYTES, bar, policy);
       }
       __syncwarp();
       if (ok) {
@@ -389,21 +399,38 @@ __global__ void __launch_bounds__(kThreads, SB == 4096 ? 4 : 2) decode_attn_kern
     ++pseq;
     ++px;
     advance(pc, pre, B, Hkv);
-    if (px == pend) {  // chunk finished: move to the chunk requested ahead
+  };
+  // Issue the next stage; when the current chunk is used up, first move on
+  // to the chunk requested ahead (the consumer follows through
+  // chunk_for_consumer: the switch always happens before the consumer has
+  // finished the previous chunk, because that chunk's stages were all issued
+  // at least one consumer step earlier).
+  auto producer_step = [&]() {
+    if (p_done) return;
+    if (px == pend) {
       p_chunk = grab_take();
       chunk_for_consumer = p_chunk;
-      if (p_chunk < nchunks) {
-        px = chunk_begin(p_chunk);
-        pend = chunk_end_x(p_chunk);
-        pc = locate(px, pre, B, Hkv);
-        grab_issue();
-      } else {
+      if (p_chunk >= nchunks) {
         p_done = true;
+        return;
       }
+      px = chunk_begin(p_chunk);
+      pend = chunk_end_x(p_chunk);
+      pc = locate(px, pre, B, Hkv);
+      grab_issue();
     }
+    issue();
   };
 
-  for (int s = 0; s < kWStages && !p_done; ++s) issue();
+  const Cursor pc0 = pc;  // first piece of this warp
+  for (int s = 0; s < kWStages && !p_done && px < pend; ++s) issue();
+  if (early) asm volatile("griddepcontrol.wait;" ::: "memory");
+  if (lane == 0) {
+    mbar_arrive_expect_tx(&qbars[warp], Q_BYTES);
+    bulk_g2s(myq, reinterpret_cast<const T*>(p.q) + ((int64_t)pc0.b * p.Hq + pc0.h * G) * HD,
+             Q_BYTES, &qbars[warp], policy);
+  }
+  grab_issue();  // the next chunk, requested one ahead
 
   // ---- consumer
   const int log2P_in_stage = p.P >= STAGE_SLOTS ? 30 : p.log2P;  // stage page index = slot >> this
@@ -417,12 +444,14 @@ __global__ void __launch_bounds__(kThreads, SB == 4096 ? 4 : 2) decode_attn_kern
   T* outp = reinterpret_cast<T*>(p.out);
   for (uint32_t seq = 0;; ++seq) {
     const int buf = (int)(seq % kWStages);
-    const bool ok = mbar_wait(&bars[warp][buf], (seq / kWStages) & 1);
+    bool ok = mbar_wait(&bars[warp][buf], (seq / kWStages) & 1);
+    if (seq == 0) ok = mbar_wait(&qbars[warp], 0) && ok;  // the first piece's query
     if (__any_sync(FULLMASK, !ok)) {
       // a copy never landed: report, drain what is in flight (bounded) and stop
       if (lane == 0) {
         report(p.status, WM_ERR_TIMEOUT);
         for (uint32_t y = seq; y < pseq; ++y) mbar_wait(&bars[warp][y % kWStages], (y / kWStages) & 1);
+        if (seq == 0) mbar_wait(&qbars[warp], 0);
       }
       __syncwarp();
       return;
@@ -449,7 +478,7 @@ __global__ void __launch_bounds__(kThreads, SB == 4096 ? 4 : 2) decode_attn_kern
       consume_stage<T, HD, G, SB, false>(Ks, Vs, lane_slot, lane_part, q2, p.qscale, valid_slots,
                                          mask, log2P_in_stage, st);
     __syncwarp();  // every lane is done with this ring slot
-    if (!p_done) issue();
+    producer_step();
 
     const bool chunk_end = (cx == cend - 1);
     if (chunk_end || cc.st == cc.nst - 1) {
@@ -566,6 +595,7 @@ __global__ void __launch_bounds__(kThreads, SB == 4096 ? 4 : 2) decode_attn_kern
       piece_first = false;
     }
     if (chunk_end) {  // continue with the chunk the producer moved on to
+      if (chunk_for_consumer < 0) producer_step();  // a chunk shorter than the ring
       c_chunk = chunk_for_consumer;
       if (c_chunk < 0 || c_chunk >= nchunks) break;
       cx = chunk_begin(c_chunk);

@@ -22,8 +22,9 @@ struct AttnParams {
   int32_t* status;
   int64_t page_stride;    // elements between consecutive physical pages
   int32_t B, Hq, Hkv, P, log2P, num_pages, max_pages;
-  int32_t chunk_stages;   // stages per work chunk
+  int32_t chunk_stages;   // stages per work chunk (0: one chunk per warp)
   int32_t max_chunks;     // partial slots per side
+  int32_t inputs_ready;   // the previous grid wrote no cache, table, length or workspace
   float qscale;           // log2(e) / sqrt(d)
 };
 

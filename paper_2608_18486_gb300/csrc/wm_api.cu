@@ -170,7 +170,17 @@ wm_status wm_decode_attn(const wm_config* c, const wm_cache* cache, int32_t laye
                          const int32_t* page_table, const int32_t* seq_lens, int32_t B,
                          int32_t max_pages, void* out, void* workspace, size_t ws_bytes,
                          int32_t* dev_status, void* stream) {
+  return wm_decode_attn_flags(c, cache, layer, q, page_table, seq_lens, B, max_pages, out,
+                              workspace, ws_bytes, 0u, dev_status, stream);
+}
+
+wm_status wm_decode_attn_flags(const wm_config* c, const wm_cache* cache, int32_t layer,
+                               const void* q, const int32_t* page_table, const int32_t* seq_lens,
+                               int32_t B, int32_t max_pages, void* out, void* workspace,
+                               size_t ws_bytes, uint32_t flags, int32_t* dev_status, void* stream) {
   wm_status st = wm_config_check(c);
+  if (st != WM_OK) return st;
+  if (flags & ~(uint32_t)WM_ATTN_INPUTS_READY) return WM_ERR_INVALID_ARG;
   if (st != WM_OK) return st;
   if ((st = check_cache(*c, cache)) != WM_OK) return st;
   if (layer < 0 || layer >= c->L || B < 0 || max_pages < 1) return WM_ERR_INVALID_ARG;
@@ -206,6 +216,7 @@ wm_status wm_decode_attn(const wm_config* c, const wm_cache* cache, int32_t laye
   p.B = B;
   p.chunk_stages = pl.chunk_stages;
   p.max_chunks = pl.max_chunks;
+  p.inputs_ready = (flags & WM_ATTN_INPUTS_READY) ? 1 : 0;
   p.qscale = (float)(1.4426950408889634 / sqrt((double)c->d));
   cudaError_t e = wm::launch_decode_attn(p, pl.stage_bytes, c->dtype, c->d, c->Hq / c->Hkv,
                                          pl.grid, (cudaStream_t)stream);

@@ -62,13 +62,16 @@ class DecodeSession:
 
     # ------------------------------------------------------------------ calls
     def decode_attn(self, layer: int, q, page_table, seq_lens, out, B: int | None = None,
-                    stream=None) -> None:
+                    stream=None, inputs_ready: bool = False) -> None:
+        """inputs_ready: the previous work on the stream wrote no cache, page
+        table, lengths or workspace (true for layers 1..L-1 of a decode step)."""
         B = self.B if B is None else B
-        rc = W.wm_decode_attn(self.cfg, self.cache, layer, q, page_table, seq_lens, B,
-                              self.max_pages, out, self.attn_ws, self.attn_ws_bytes, self.status,
-                              self._stream(stream))
+        flags = W.WM_ATTN_INPUTS_READY if inputs_ready else 0
+        rc = W.wm_decode_attn_flags(self.cfg, self.cache, layer, q, page_table, seq_lens, B,
+                                    self.max_pages, out, self.attn_ws, self.attn_ws_bytes, flags,
+                                    self.status, self._stream(stream))
         if rc != W.WM_OK:
-            raise W.WMError(rc, "wm_decode_attn")
+            raise W.WMError(rc, "wm_decode_attn_flags")
 
     def kv_mix(self, h, page_table, slot, B: int | None = None, stream=None) -> None:
         if self._weights is None:

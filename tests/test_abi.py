@@ -86,6 +86,8 @@ def test_compute_calls_reject_bad_arguments_before_launching():
     # a cache laid out for another config is refused
     other = cfg(k=8)
     assert W.wm_decode_attn(other, cache, 0, fake, fake, fake, 2, 4, fake, fake, ws, None, None) == W.WM_ERR_INVALID_ARG
+    assert W.wm_decode_attn_flags(c, cache, 0, fake, fake, fake, 2, 4, fake, fake, ws, 2, None,
+                                  None) == W.WM_ERR_INVALID_ARG  # unknown flag bit
     wts = W.mix_weights((fake, fake), (fake, fake), (fake, fake), (fake, fake), (fake, fake), fake)
     mws = W.wm_kv_mix_workspace(c, 2)
     assert W.wm_kv_mix(c, cache, wts, fake, fake, fake, 2, 4, fake, mws - 1, None, None) == W.WM_ERR_INVALID_ARG

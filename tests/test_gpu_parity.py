@@ -225,3 +225,24 @@ def test_device_generator_matches_host_bit_for_bit():
                                                                  0.37, 1.0))
         got = t.cpu().view(torch.int32 if dtype == "f32" else torch.int16).numpy()
         assert np.array_equal(got, host.view(np.int32 if dtype == "f32" else np.int16))
+
+
+@pytest.mark.parametrize("name,overrides", [("no_compression", dict()),
+                                            ("large", dict(k=1, B=4))])
+def test_inputs_ready_chain_matches_default_launches(name, overrides):
+    """Layers 1..L-1 launched with WM_ATTN_INPUTS_READY (K/V fetched while the
+    previous launch finishes) give the same bits as plain launches."""
+    w = configs.get(name).with_(**overrides)
+    prob, sess, dp = H.setup(w)
+    ref = [H.run_attn(sess, dp, l).clone() for l in range(w.L)]
+    outs = torch.empty((w.L, w.B, w.Hq, w.d), dtype=sess.dtype, device="cuda")
+    for _ in range(2):
+        for l in range(w.L):
+            sess.decode_attn(l, dp.q[l], dp.page_table, dp.seq_lens, outs[l], inputs_ready=l > 0)
+    torch.cuda.synchronize()
+    assert sess.read_status() == 0
+    for l in range(w.L):
+        assert torch.equal(outs[l], ref[l]), l
+    if name == "no_compression":
+        assert H.rel_err(H.to_f64(outs[3]), H.oracle_attn_full(prob, 3)) <= H.TOL[w.dtype]
+    _free()

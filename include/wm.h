@@ -56,7 +56,7 @@ extern "C" {
 typedef enum {
   WM_OK = 0,
   WM_ERR_INVALID_ARG = 1, /* bad pointer, size or configuration value        */
-  WM_ERR_UNSUPPORTED = 2, /* valid per the paper, not built here (e.g. d=96) */
+  WM_ERR_UNSUPPORTED = 2, /* valid per the paper, not built here (e.g. d=80) */
   WM_ERR_CUDA = 3,        /* a CUDA runtime call or launch failed            */
   WM_ERR_BOUNDS = 4,      /* device: page id, slot or length out of range    */
   WM_ERR_TIMEOUT = 5      /* device: a bounded pipeline wait ran out         */
@@ -71,7 +71,7 @@ typedef struct {
   int32_t D;          /* hidden width; multiple of 8, at most 4096                 */
   int32_t Hq;         /* query heads; multiple of Hkv, Hq/Hkv in {1,2,4,8}         */
   int32_t Hkv;        /* key/value heads per channel                               */
-  int32_t d;          /* head dimension: 64 or 128                                 */
+  int32_t d;          /* head dimension: 64, 96 or 128                             */
   int32_t p;          /* router reads every p-th layer from L-1 down, p >= 1       */
   int32_t page_size;  /* cache slots per page: a power of two, 1..4096             */
   int32_t dtype;      /* wm_dtype                                                  */
@@ -203,6 +203,17 @@ wm_status wm_decode_attn_flags(const wm_config* cfg, const wm_cache* cache, int3
                                const int32_t* seq_lens, int32_t B, int32_t max_pages, void* out,
                                void* workspace, size_t ws_bytes, uint32_t flags,
                                int32_t* dev_status, void* stream);
+
+/*
+ * Self-test of the kernels' failure detection (no counterpart in the paper).
+ * Every pipeline wait in this library is bounded; when a wait runs out the
+ * kernel writes WM_ERR_TIMEOUT to the status word and returns instead of
+ * hanging.  This launches one block that waits on a barrier that nothing
+ * will complete, with a limit of limit_us microseconds (1 .. 2,000,000), so a
+ * caller can check on its GPU that the status comes back and the context
+ * stays usable.  dev_status: device int32, as for the other entry points.
+ */
+wm_status wm_selftest_bounded_wait(int32_t* dev_status, uint32_t limit_us, void* stream);
 
 /*
  * Decode attention for callers that cannot allocate device memory.

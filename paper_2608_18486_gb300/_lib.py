@@ -181,3 +181,11 @@ def wm_decode_attn_noalloc(cfg, cache, layer, q, page_table, seq_lens, B, max_pa
     return L.wm_decode_attn_noalloc(ctypes.byref(cfg), ctypes.byref(cache), int(layer), _p(q),
                                     _p(page_table), _p(seq_lens), int(B), int(max_pages), _p(out),
                                     _p(dev_status), stream)
+
+
+def wm_selftest_bounded_wait(dev_status, limit_us: int, stream) -> int:
+    """Run the bounded-wait self-test (see include/wm.h)."""
+    L = lib()
+    L.wm_selftest_bounded_wait.restype = ctypes.c_int
+    L.wm_selftest_bounded_wait.argtypes = [ctypes.c_void_p, ctypes.c_uint32, ctypes.c_void_p]
+    return L.wm_selftest_bounded_wait(_p(dev_status), int(limit_us), stream)

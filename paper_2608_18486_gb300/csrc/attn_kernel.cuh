@@ -1,0 +1,661 @@
+#pragma once
+// Decode attention over one channel of the paged k-channel cache
+// (Sec. 3.1 Step 3; dummy slot of Sec. 3.2).
+//
+// Design (GB300).  The work is a stream over the KV blocks of every
+// (sequence b, kv head h) unit of the chosen channel; it reads about one byte
+// per FLOP, so it is HBM-bound and runs on the CUDA cores.
+//
+//  * Stream-K split.  Each unit is cut into pipeline stages of STAGE_SLOTS
+//    slots (4 or 8 KB of K+V).  The stages of all units, concatenated, are
+//    cut into equal chunks of CH stages.  Warp w of the persistent grid
+//    starts on chunk w and then takes further chunks from an atomic counter
+//    (requested one chunk ahead), so warps that stream faster take more
+//    chunks and all finish together whatever the sequence lengths.
+//  * Private pipelines.  Each warp owns a 3-deep ring in shared memory and
+//    fills it with 1-D bulk async copies (TMA engine, mbarrier completion,
+//    L2 evict-first) of contiguous (page, kv-head) runs; it refills a slot as
+//    soon as it has consumed it, so no block-wide barrier is ever taken.
+//  * Compute.  8 lanes own one slot (16-byte vectors, conflict-free shared
+//    loads), reduce q.k with xor shuffles and keep an online softmax
+//    (running max m, sum l, accumulator) per lane group; groups merge with
+//    shuffles at the end of a piece.
+//  * Merge.  A piece of a unit that lies inside one chunk is written straight
+//    to the output.  Only units that cross a chunk boundary leave partials
+//    (at most two per chunk: its first and its last piece); the last warp to
+//    finish such a unit (atomic ticket, no waiting) merges them.
+#include <math.h>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace wm {
+namespace attn_detail {
+
+constexpr int kWarps = 4;
+constexpr int kThreads = kWarps * 32;
+constexpr int kWStages = 3;          // ring depth per warp
+
+// Largest power of two <= x (x >= 1).
+constexpr int pow2_floor(int x) { return x >= 2 ? 2 * pow2_floor(x / 2) : 1; }
+
+// SB: K + V byte budget of one pipeline stage (4 KB or 8 KB).
+template <typename T, int HD, int SB>
+struct Shape {
+  // A slot row is ROW_VECS 16-byte vectors.  LPS lanes own one slot, lane
+  // part p holding vectors p, p + LPS, ...; with 8 lanes a quarter warp reads
+  // one contiguous 128-byte run, with 4 lanes (rows of 12 vectors, d = 96
+  // bf16) it reads 64 bytes from each of two rows 192 bytes apart, which
+  // fall on disjoint banks.  Either way every 16-byte shared load of the
+  // warp is bank-conflict free.
+  static constexpr int VEC = Elem<T>::kVec;                       // elements per 16 bytes
+  static constexpr int ROW_VECS = HD * (int)sizeof(T) / 16;
+  static constexpr int LPS = ROW_VECS % 8 == 0 ? 8 : 4;           // lanes per slot
+  static constexpr int SPW = 32 / LPS;                            // slots per warp step
+  static constexpr int NVL = ROW_VECS / LPS;                      // 16-byte vectors per lane
+  static constexpr int EPL = NVL * VEC;                           // elements per lane
+  static constexpr int STAGE_SLOTS = pow2_floor(SB / (2 * HD * (int)sizeof(T)));
+  static constexpr int STAGE_ELEMS = STAGE_SLOTS * HD;
+  static constexpr int ITERS = STAGE_SLOTS / SPW;
+  static_assert(ROW_VECS % LPS == 0 && NVL >= 1, "lane split");
+  static_assert(ITERS >= 1 && STAGE_SLOTS % SPW == 0 && STAGE_SLOTS <= 32, "stage split");
+};
+
+// Lane part `lp` owns the 16-byte vectors lp, lp + 8, ... of a slot row.
+template <typename T, int HD, int SB>
+__device__ __forceinline__ void load_row(const T* row, int lp, float2 (&f)[Shape<T, HD, SB>::EPL / 2]) {
+  using SH = Shape<T, HD, SB>;
+#pragma unroll
+  for (int v = 0; v < SH::NVL; ++v) {
+    float t[SH::VEC];
+    Elem<T>::unpack(*reinterpret_cast<const uint4*>(row + (v * SH::LPS + lp) * SH::VEC), t);
+#pragma unroll
+    for (int i = 0; i < SH::VEC / 2; ++i) f[v * SH::VEC / 2 + i] = make_float2(t[2 * i], t[2 * i + 1]);
+  }
+}
+
+template <typename T>
+__device__ __forceinline__ void store_vec(T* dst, const float* v);
+template <>
+__device__ __forceinline__ void store_vec<float>(float* dst, const float* v) {
+  *reinterpret_cast<float4*>(dst) = make_float4(v[0], v[1], v[2], v[3]);
+}
+template <>
+__device__ __forceinline__ void store_vec<__nv_bfloat16>(__nv_bfloat16* dst, const float* v) {
+  uint4 u;
+  __nv_bfloat162 t;
+  t = __floats2bfloat162_rn(v[0], v[1]); u.x = *reinterpret_cast<uint32_t*>(&t);
+  t = __floats2bfloat162_rn(v[2], v[3]); u.y = *reinterpret_cast<uint32_t*>(&t);
+  t = __floats2bfloat162_rn(v[4], v[5]); u.z = *reinterpret_cast<uint32_t*>(&t);
+  t = __floats2bfloat162_rn(v[6], v[7]); u.w = *reinterpret_cast<uint32_t*>(&t);
+  *reinterpret_cast<uint4*>(dst) = u;
+}
+
+// Position in the stage stream: sequence b, kv head h, stage st of nst.
+struct Cursor {
+  int b, h, st, nst;
+};
+
+__device__ __forceinline__ Cursor locate(int64_t x, const int* pre, int B, int Hkv) {
+  int lo = 0, hi = B;  // largest b with Hkv * pre[b] <= x
+  while (hi - lo > 1) {
+    const int mid = (lo + hi) >> 1;
+    if ((int64_t)Hkv * pre[mid] <= x) lo = mid; else hi = mid;
+  }
+  Cursor c;
+  c.b = lo;
+  c.nst = pre[lo + 1] - pre[lo];
+  const int64_t r = x - (int64_t)Hkv * pre[lo];
+  c.h = (int)(r / c.nst);
+  c.st = (int)(r % c.nst);
+  return c;
+}
+
+__device__ __forceinline__ void advance(Cursor& c, const int* pre, int B, int Hkv) {
+  if (++c.st < c.nst) return;
+  c.st = 0;
+  if (++c.h < Hkv) return;
+  c.h = 0;
+  do { ++c.b; } while (c.b < B && pre[c.b + 1] == pre[c.b]);
+  if (c.b < B) c.nst = pre[c.b + 1] - pre[c.b];
+}
+
+
+// Online-softmax state of one lane: G query heads, EPL output elements each.
+template <typename T, int HD, int G, int SB>
+struct SoftState {
+  float m[G], l[G];
+  float2 acc[G][Shape<T, HD, SB>::EPL / 2];
+};
+
+// One pipeline stage of K/V rows for this warp's current piece.  FULL: every
+// slot of the stage is inside the sequence and on a fetched page, so no
+// masking is needed; otherwise masked slots never touch the sums (NaN-safe).
+template <typename T, int HD, int G, int SB, bool FULL>
+__device__ __forceinline__ void consume_stage(const T* Ks, const T* Vs, int lane_slot, int lane_part,
+                                              const float2 (&q2)[G][Shape<T, HD, SB>::EPL / 2],
+                                              float qscale, int valid_slots, uint64_t mask,
+                                              int log2P_in_stage, SoftState<T, HD, G, SB>& st) {
+  using SH = Shape<T, HD, SB>;
+  constexpr int SPW = SH::SPW, ITERS = SH::ITERS, E2 = SH::EPL / 2;
+  float sc[G][ITERS];
+#pragma unroll
+  for (int it = 0; it < ITERS; ++it) {
+    const int ls = it * SPW + lane_slot;
+    float2 kf[E2];
+    load_row<T, HD, SB>(Ks + ls * HD, lane_part, kf);
+    bool valid = true;
+    if (!FULL) valid = (ls < valid_slots) && ((mask >> (ls >> log2P_in_stage)) & 1ull);
+#pragma unroll
+    for (int g = 0; g < G; ++g) {
+      float2 a = make_float2(0.f, 0.f);
+#pragma unroll
+      for (int i = 0; i < E2; ++i) a = __ffma2_rn(q2[g][i], kf[i], a);
+      float s = group_sum<SH::LPS>(a.x + a.y) * qscale;
+      sc[g][it] = valid ? s : -INFINITY;
+    }
+  }
+#pragma unroll
+  for (int g = 0; g < G; ++g) {
+    float mx = sc[g][0];
+#pragma unroll
+    for (int it = 1; it < ITERS; ++it) mx = fmaxf(mx, sc[g][it]);
+    const float mnew = fmaxf(st.m[g], mx);
+    if (FULL || mnew != -INFINITY) {
+      const float corr = exp2f(st.m[g] - mnew);  // 0 while m is still -inf
+      st.l[g] *= corr;
+      const float2 c2 = make_float2(corr, corr);
+#pragma unroll
+      for (int i = 0; i < E2; ++i) st.acc[g][i] = __fmul2_rn(st.acc[g][i], c2);
+      st.m[g] = mnew;
+    }
+  }
+#pragma unroll
+  for (int it = 0; it < ITERS; ++it) {
+    const int ls = it * SPW + lane_slot;
+    float2 vf[E2];
+    load_row<T, HD, SB>(Vs + ls * HD, lane_part, vf);
+#pragma unroll
+    for (int g = 0; g < G; ++g) {
+      if (FULL || sc[g][it] != -INFINITY) {
+        const float pr = exp2f(sc[g][it] - st.m[g]);
+        st.l[g] += pr;
+        const float2 p2 = make_float2(pr, pr);
+#pragma unroll
+        for (int i = 0; i < E2; ++i) st.acc[g][i] = __ffma2_rn(p2, vf[i], st.acc[g][i]);
+      }
+    }
+  }
+}
+
+// Write G rows of d outputs (lanes of slot group 0 own vectors lane, lane+8, ...).
+template <typename T, int HD, int G, int SB>
+__device__ __forceinline__ void write_rows(T* out_rows, int lane_part, const SoftState<T, HD, G, SB>& st) {
+  using SH = Shape<T, HD, SB>;
+#pragma unroll
+  for (int g = 0; g < G; ++g) {
+    const float inv = st.l[g] > 0.f ? 1.f / st.l[g] : 0.f;
+#pragma unroll
+    for (int v = 0; v < SH::NVL; ++v) {
+      float o[SH::VEC];
+#pragma unroll
+      for (int i = 0; i < SH::VEC / 2; ++i) {
+        o[2 * i] = st.acc[g][v * SH::VEC / 2 + i].x * inv;
+        o[2 * i + 1] = st.acc[g][v * SH::VEC / 2 + i].y * inv;
+      }
+      store_vec<T>(out_rows + g * HD + (v * SH::LPS + lane_part) * SH::VEC, o);
+    }
+  }
+}
+
+template <typename T, int HD, int G, int SB>
+__global__ void __launch_bounds__(kThreads, attn_ctas_per_sm(SB, G)) decode_attn_kernel(const AttnParams p) {
+  using SH = Shape<T, HD, SB>;
+  constexpr int VEC = SH::VEC, LPS = SH::LPS, E2 = SH::EPL / 2;
+  constexpr int STAGE_SLOTS = SH::STAGE_SLOTS, STAGE_ELEMS = SH::STAGE_ELEMS;
+  constexpr uint32_t KV_BYTES = STAGE_ELEMS * sizeof(T);
+  constexpr uint32_t Q_BYTES = G * HD * sizeof(T);
+  constexpr unsigned FULLMASK = 0xFFFFFFFFu;
+
+  extern __shared__ __align__(128) unsigned char smem_raw[];
+  T* ring = reinterpret_cast<T*>(smem_raw);                       // [W][S][2][STAGE_ELEMS]
+  T* qring = ring + kWarps * kWStages * 2 * STAGE_ELEMS;          // [W][S][G*HD]
+  int* pre = reinterpret_cast<int*>(qring + kWarps * kWStages * G * HD);  // [B+1]
+  int* lens = pre + p.B + 1;                                      // [B]
+  __shared__ uint64_t bars[kWarps][kWStages];
+  __shared__ uint64_t qbars[kWarps];  // query of the warp's first piece
+  __shared__ uint64_t masks[kWarps][kWStages];
+  __shared__ int scan[kThreads];
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int B = p.B, Hkv = p.Hkv;
+  const int max_slots = p.max_pages * p.P;
+
+  // Programmatic dependent launch: the next grid on the stream may be
+  // scheduled now.  This grid waits for the previous one (finished and
+  // flushed) before reading anything it may have written.  With the caller's
+  // promise that the previous grid wrote neither the cache, the page table,
+  // the lengths nor the workspace (inputs_ready), the wait moves down to just
+  // before the query is read, and the first K/V copies overlap its tail.
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  const bool early = p.inputs_ready != 0;
+  if (!early) asm volatile("griddepcontrol.wait;" ::: "memory");
+
+  // ---- stages per sequence and their prefix sums (every CTA, all threads)
+  {
+    const int per = (B + kThreads - 1) / kThreads;
+    const int i0 = min(B, tid * per), i1 = min(B, i0 + per);
+    int sum = 0;
+    for (int i = i0; i < i1; ++i) {
+      const int S = p.seq_lens[i];
+      const bool ok = S >= 1 && S <= max_slots;
+      lens[i] = ok ? S : 0;
+      sum += ok ? (S + STAGE_SLOTS - 1) / STAGE_SLOTS : 0;
+    }
+    scan[tid] = sum;
+    __syncthreads();
+    for (int o = 1; o < kThreads; o <<= 1) {  // inclusive Hillis-Steele scan
+      const int v = tid >= o ? scan[tid - o] : 0;
+      __syncthreads();
+      scan[tid] += v;
+      __syncthreads();
+    }
+    int run = scan[tid] - sum;
+    for (int i = i0; i < i1; ++i) {
+      pre[i] = run;
+      run += lens[i] ? (lens[i] + STAGE_SLOTS - 1) / STAGE_SLOTS : 0;
+    }
+    if (tid == kThreads - 1) pre[B] = scan[tid];
+    if (lane == 0) {
+      for (int s = 0; s < kWStages; ++s) mbar_init(&bars[warp][s], 1);
+      mbar_init(&qbars[warp], 1);
+    }
+    fence_mbar_init();
+    __syncthreads();
+  }
+  // ---- sequences with an invalid length: zero output rows, report once
+  if (blockIdx.x == 0) {
+    if (early) asm volatile("griddepcontrol.wait;" ::: "memory");
+    for (int b = 0; b < B; ++b) {
+      if (lens[b] != 0) continue;
+      T* o = reinterpret_cast<T*>(p.out) + (int64_t)b * p.Hq * HD;
+      for (int i = tid; i < p.Hq * HD; i += kThreads) o[i] = Elem<T>::from_f(0.f);
+      if (tid == 0) report(p.status, WM_ERR_BOUNDS);
+    }
+  }
+
+  // The NS stages split into nchunks near-equal chunks [c*NS/n, (c+1)*NS/n).
+  // Every chunk has at least CH > kWStages stages, so the producer, at most
+  // kWStages stages ahead, is never more than one chunk ahead of the consumer.
+  // chunk_stages == 0: static split, one chunk per warp and no chunk counter.
+  const int64_t NS = (int64_t)Hkv * pre[B];  // stages of all units, concatenated
+  const int64_t GW = (int64_t)gridDim.x * kWarps;
+  const bool dynamic = p.chunk_stages > 0;
+  const int64_t CH = dynamic ? p.chunk_stages : (int64_t)kWStages + 1;
+  int64_t nchunks = NS / CH > 1 ? NS / CH : 1;
+  if (!dynamic && nchunks > GW) nchunks = GW;
+  auto chunk_begin = [&](int64_t c) -> int64_t { return c * NS / nchunks; };
+  auto chunk_end_x = [&](int64_t c) -> int64_t { return (c + 1) * NS / nchunks; };
+  auto chunk_of = [&](int64_t x) -> int64_t { return ((x + 1) * nchunks - 1) / NS; };
+  const int64_t gw = (int64_t)blockIdx.x * kWarps + warp;
+  int32_t* grab_ctr = p.counters + (int64_t)B * Hkv;
+  // Every warp ends with exactly one request that finds no chunk; the request
+  // that is last of all resets the counter for the next launch.  A request is
+  // issued one chunk ahead and its result read only when the chunk is needed.
+  const int64_t total_grabs = (nchunks > GW ? nchunks - GW : 0) + GW;
+  int grab_t = 0;  // lane 0: counter value of the outstanding request
+  auto grab_issue = [&]() {
+    if (dynamic && lane == 0) grab_t = atomicAdd(grab_ctr, 1);
+  };
+  auto grab_take = [&]() -> int64_t {
+    if (!dynamic) return nchunks;  // static split: no further chunk
+    if (lane == 0 && grab_t == total_grabs - 1) atomicExch(grab_ctr, 0);
+    return GW + __shfl_sync(FULLMASK, grab_t, 0);
+  };
+  if (gw >= nchunks || NS == 0) {
+    if (early) asm volatile("griddepcontrol.wait;" ::: "memory");
+    grab_issue();
+    grab_take();
+    return;  // warp-level from here on: no block barriers below
+  }
+
+  T* myring = ring + warp * kWStages * 2 * STAGE_ELEMS;
+  T* myq = qring + warp * kWStages * G * HD;
+  const uint64_t policy = l2_evict_first_policy();
+  const int lane_slot = lane / LPS, lane_part = lane % LPS;
+
+  // ---- page-table window of the producer: lane i holds the page id of
+  // logical page win0 + i (cur) and win0 + 32 + i (nxt) of sequence win_b.
+  int win_b = -1, win0 = 0, pg_cur = -1, pg_nxt = -1;
+  auto load_pg = [&](int b, int lp) -> int {
+    return lp < p.max_pages ? __ldg(p.page_table + (int64_t)b * p.max_pages + lp) : -1;
+  };
+  // page id of logical page lp + (this lane's offset) -- all lanes call it together
+  auto page_of = [&](int b, int lp, int lane_off) -> int {
+    if (b != win_b || lp < win0 || lp >= win0 + 64) {
+      win_b = b;
+      win0 = lp;
+      pg_cur = load_pg(b, lp + lane);
+      pg_nxt = load_pg(b, lp + 32 + lane);
+    } else if (lp >= win0 + 32) {
+      win0 += 32;
+      pg_cur = pg_nxt;
+      pg_nxt = load_pg(b, win0 + 32 + lane);
+    }
+    const int idx = lp + lane_off - win0;  // 0 .. 63
+    const int a = __shfl_sync(FULLMASK, pg_cur, idx & 31);
+    const int c = __shfl_sync(FULLMASK, pg_nxt, idx & 31);
+    return idx < 32 ? a : c;
+  };
+
+  // ---- producer: walks its chunks stage by stage, kWStages ahead of the consumer
+  int64_t p_chunk = gw;
+  int64_t px = chunk_begin(p_chunk), pend = chunk_end_x(p_chunk);
+  int64_t chunk_for_consumer = -1;              // the producer's chunk after a switch
+  bool p_done = false;
+  Cursor pc = locate(px, pre, B, Hkv);
+  uint32_t pseq = 0;                            // stages issued
+  auto issue = [&]() {
+    const int buf = (int)(pseq % kWStages);
+    const bool first = (px == chunk_begin(p_chunk)) || pc.st == 0;
+    const int S = lens[pc.b];
+    const int s_begin = pc.st * STAGE_SLOTS;
+    const T* kb = reinterpret_cast<const T*>(p.k_pool) + (int64_t)pc.h * p.P * HD;
+    const T* vb = reinterpret_cast<const T*>(p.v_pool) + (int64_t)pc.h * p.P * HD;
+    T* kd = myring + buf * 2 * STAGE_ELEMS;
+    T* vd = kd + STAGE_ELEMS;
+    uint64_t* bar = &bars[warp][buf];
+    // the first piece's query arrives on qbars (issued after the dependency wait)
+    const bool with_q = first && pseq > 0;
+    const uint32_t qb = with_q ? Q_BYTES : 0u;
+    const T* qsrc = reinterpret_cast<const T*>(p.q) + ((int64_t)pc.b * p.Hq + pc.h * G) * HD;
+    if (p.P >= STAGE_SLOTS) {
+      const int pg = page_of(pc.b, s_begin >> p.log2P, 0);
+      if (lane == 0) {
+        const bool ok = pg >= 0 && pg < p.num_pages;
+        masks[warp][buf] = ok ? 1ull : 0ull;
+        if (!ok) report(p.status, WM_ERR_BOUNDS);
+        mbar_arrive_expect_tx(bar, (ok ? 2 * KV_BYTES : 0u) + qb);
+        if (ok) {
+          const int64_t off = (int64_t)pg * p.page_stride + (int64_t)(s_begin & (p.P - 1)) * HD;
+          bulk_g2s(kd, kb + off, KV_BYTES, bar, policy);
+          bulk_g2s(vd, vb + off, KV_BYTES, bar, policy);
+        }
+        if (with_q) bulk_g2s(myq + buf * G * HD, qsrc, Q_BYTES, bar, policy);
+      }
+    } else {
+      const int npp = STAGE_SLOTS >> p.log2P;  // pages per stage (<= 32)
+      const int lp0 = s_begin >> p.log2P;
+      const int lpn = min(npp, ((S - 1) >> p.log2P) - lp0 + 1);
+      const int pg = page_of(pc.b, lp0, lane < lpn ? lane : 0);
+      const bool ok = lane < lpn && pg >= 0 && pg < p.num_pages;
+      const uint32_t mask = __ballot_sync(FULLMASK, ok);
+      const uint32_t bytes = (uint32_t)p.P * HD * sizeof(T);
+      if (lane == 0) {
+        masks[warp][buf] = mask;
+        if (__popc(mask) < lpn) report(p.status, WM_ERR_BOUNDS);
+        mbar_arrive_expect_tx(bar, 2u * bytes * (uint32_t)__popc(mask) + qb);
+        if (with_q) bulk_g2s(myq + buf * G * HD, qsrc, Q_BYTES, bar, policy);
+      }
+      __syncwarp();
+      if (ok) {
+        const int64_t off = (int64_t)pg * p.page_stride;
+        bulk_g2s(kd + lane * p.P * HD, kb + off, bytes, bar, policy);
+        bulk_g2s(vd + lane * p.P * HD, vb + off, bytes, bar, policy);
+      }
+    }
+    ++pseq;
+    ++px;
+    advance(pc, pre, B, Hkv);
+  };
+  // Issue the next stage; when the current chunk is used up, first move on
+  // to the chunk requested ahead (the consumer follows through
+  // chunk_for_consumer: the switch always happens before the consumer has
+  // finished the previous chunk, because that chunk's stages were all issued
+  // at least one consumer step earlier).
+  auto producer_step = [&]() {
+    if (p_done) return;
+    if (px == pend) {
+      p_chunk = grab_take();
+      chunk_for_consumer = p_chunk;
+      if (p_chunk >= nchunks) {
+        p_done = true;
+        return;
+      }
+      px = chunk_begin(p_chunk);
+      pend = chunk_end_x(p_chunk);
+      pc = locate(px, pre, B, Hkv);
+      grab_issue();
+    }
+    issue();
+  };
+
+  const Cursor pc0 = pc;  // first piece of this warp
+  for (int s = 0; s < kWStages && !p_done && px < pend; ++s) issue();
+  if (early) asm volatile("griddepcontrol.wait;" ::: "memory");
+  if (lane == 0) {
+    mbar_arrive_expect_tx(&qbars[warp], Q_BYTES);
+    bulk_g2s(myq, reinterpret_cast<const T*>(p.q) + ((int64_t)pc0.b * p.Hq + pc0.h * G) * HD,
+             Q_BYTES, &qbars[warp], policy);
+  }
+  grab_issue();  // the next chunk, requested one ahead
+
+  // ---- consumer
+  const int log2P_in_stage = p.P >= STAGE_SLOTS ? 30 : p.log2P;  // stage page index = slot >> this
+  const uint64_t all_pages = p.P >= STAGE_SLOTS ? 1ull : ((1ull << (STAGE_SLOTS >> p.log2P)) - 1ull);
+  int64_t c_chunk = gw;
+  int64_t cx = chunk_begin(c_chunk), cend = chunk_end_x(c_chunk);
+  Cursor cc = locate(cx, pre, B, Hkv);
+  bool piece_first = true;  // the current piece starts at its chunk's first stage
+  float2 q2[G][E2];
+  SoftState<T, HD, G, SB> st;
+  T* outp = reinterpret_cast<T*>(p.out);
+  for (uint32_t seq = 0;; ++seq) {
+    const int buf = (int)(seq % kWStages);
+    bool ok = mbar_wait(&bars[warp][buf], (seq / kWStages) & 1);
+    if (seq == 0) ok = mbar_wait(&qbars[warp], 0) && ok;  // the first piece's query
+    if (__any_sync(FULLMASK, !ok)) {
+      // a copy never landed: report, drain what is in flight (bounded) and stop
+      if (lane == 0) {
+        report(p.status, WM_ERR_TIMEOUT);
+        for (uint32_t y = seq; y < pseq; ++y) mbar_wait(&bars[warp][y % kWStages], (y / kWStages) & 1);
+        if (seq == 0) mbar_wait(&qbars[warp], 0);
+      }
+      __syncwarp();
+      return;
+    }
+    if (cx == chunk_begin(c_chunk) || cc.st == 0) {
+      const T* qs = myq + buf * G * HD;
+#pragma unroll
+      for (int g = 0; g < G; ++g) {
+        load_row<T, HD, SB>(qs + g * HD, lane_part, q2[g]);
+        st.m[g] = -INFINITY;
+        st.l[g] = 0.f;
+#pragma unroll
+        for (int i = 0; i < E2; ++i) st.acc[g][i] = make_float2(0.f, 0.f);
+      }
+    }
+    const int valid_slots = lens[cc.b] - cc.st * STAGE_SLOTS;
+    const uint64_t mask = masks[warp][buf];
+    const T* Ks = myring + buf * 2 * STAGE_ELEMS;
+    const T* Vs = Ks + STAGE_ELEMS;
+    if (valid_slots >= STAGE_SLOTS && mask == all_pages)
+      consume_stage<T, HD, G, SB, true>(Ks, Vs, lane_slot, lane_part, q2, p.qscale, valid_slots,
+                                        mask, log2P_in_stage, st);
+    else
+      consume_stage<T, HD, G, SB, false>(Ks, Vs, lane_slot, lane_part, q2, p.qscale, valid_slots,
+                                         mask, log2P_in_stage, st);
+    __syncwarp();  // every lane is done with this ring slot
+    producer_step();
+
+    const bool chunk_end = (cx == cend - 1);
+    if (chunk_end || cc.st == cc.nst - 1) {
+      // merge the SPW lane groups of the warp
+#pragma unroll
+      for (int g = 0; g < G; ++g) {
+        float M = st.m[g];
+#pragma unroll
+        for (int o = LPS; o < 32; o <<= 1) M = fmaxf(M, __shfl_xor_sync(FULLMASK, M, o));
+        const float w = (st.m[g] == -INFINITY) ? 0.f : exp2f(st.m[g] - M);
+        float Ls = st.l[g] * w;
+#pragma unroll
+        for (int o = LPS; o < 32; o <<= 1) Ls += __shfl_xor_sync(FULLMASK, Ls, o);
+#pragma unroll
+        for (int i = 0; i < E2; ++i) {
+          float2 a = __fmul2_rn(st.acc[g][i], make_float2(w, w));
+#pragma unroll
+          for (int o = LPS; o < 32; o <<= 1) {
+            a.x += __shfl_xor_sync(FULLMASK, a.x, o);
+            a.y += __shfl_xor_sync(FULLMASK, a.y, o);
+          }
+          st.acc[g][i] = a;
+        }
+        st.m[g] = M;
+        st.l[g] = Ls;
+      }
+      const int64_t rowbase = (int64_t)cc.b * p.Hq + cc.h * G;
+      const int64_t U = (int64_t)Hkv * pre[cc.b] + (int64_t)cc.h * cc.nst;
+      const int64_t g_first = chunk_of(U), g_last = chunk_of(U + cc.nst - 1);
+      if (g_first == g_last) {
+        if (lane_slot == 0) write_rows<T, HD, G, SB>(outp + rowbase * HD, lane_part, st);
+      } else {
+        // partial of this piece: its chunk's first piece -> side 0, last piece -> side 1
+        for (int side = 0; side < 2; ++side) {
+          if ((side == 0 && !piece_first) || (side == 1 && !chunk_end)) continue;
+          float* po = p.part_o + ((int64_t)side * p.max_chunks + c_chunk) * G * HD;
+          float* pm = p.part_ml + ((int64_t)side * p.max_chunks + c_chunk) * G * 2;
+          if (lane_slot == 0) {
+#pragma unroll
+            for (int g = 0; g < G; ++g)
+#pragma unroll
+              for (int v = 0; v < SH::NVL; ++v)
+#pragma unroll
+                for (int i = 0; i < VEC / 2; ++i)
+                  reinterpret_cast<float2*>(po + g * HD + (v * LPS + lane_part) * VEC)[i] =
+                      st.acc[g][v * VEC / 2 + i];
+          }
+          if (lane == 0) {
+#pragma unroll
+            for (int g = 0; g < G; ++g) {
+              pm[2 * g] = st.m[g];
+              pm[2 * g + 1] = st.l[g];
+            }
+          }
+        }
+        __threadfence();
+        __syncwarp();
+        int last = 0;
+        if (lane == 0) {
+          const int t = atomicAdd(&p.counters[cc.b * Hkv + cc.h], 1);
+          last = (t == (int)(g_last - g_first));
+        }
+        last = __shfl_sync(FULLMASK, last, 0);
+        if (last) {
+          __threadfence();
+          // merge the pieces of chunks g_first .. g_last (side 1 of the first
+          // chunk, side 0 of the others), up to 32 pieces per round, one per lane
+          const int np = (int)(g_last - g_first + 1);
+          for (int g = 0; g < G; ++g) {
+            float M = -INFINITY, Ls = 0.f;
+            float o[HD / 32];
+#pragma unroll
+            for (int i = 0; i < HD / 32; ++i) o[i] = 0.f;
+            for (int r0 = 0; r0 < np; r0 += 32) {
+              const int nr = min(32, np - r0);
+              float mq = -INFINITY, lq = 0.f;
+              if (lane < nr) {
+                const int64_t q = g_first + r0 + lane;
+                const float* pm = p.part_ml + ((int64_t)(q == g_first ? 1 : 0) * p.max_chunks + q) * G * 2 + 2 * g;
+                mq = __ldcg(pm);
+                lq = __ldcg(pm + 1);
+              }
+              float Mr = mq;
+#pragma unroll
+              for (int o2 = 16; o2 > 0; o2 >>= 1) Mr = fmaxf(Mr, __shfl_xor_sync(FULLMASK, Mr, o2));
+              const float Mn = fmaxf(M, Mr);
+              if (Mn == -INFINITY) continue;
+              const float rescale = exp2f(M - Mn);  // 0 on the first round
+              const float w = (mq == -INFINITY) ? 0.f : exp2f(mq - Mn);
+              float lw = w * lq;
+#pragma unroll
+              for (int o2 = 16; o2 > 0; o2 >>= 1) lw += __shfl_xor_sync(FULLMASK, lw, o2);
+              Ls = Ls * rescale + lw;
+#pragma unroll
+              for (int i = 0; i < HD / 32; ++i) o[i] *= rescale;
+#pragma unroll 4
+              for (int j = 0; j < nr; ++j) {
+                const float wj = __shfl_sync(FULLMASK, w, j);
+                const int64_t q = g_first + r0 + j;
+                const float* po = p.part_o + (((int64_t)(q == g_first ? 1 : 0) * p.max_chunks + q) * G + g) * HD;
+#pragma unroll
+                for (int i = 0; i < HD / 32; ++i) o[i] = fmaf(wj, __ldcg(po + lane + 32 * i), o[i]);
+              }
+              M = Mn;
+            }
+            const float inv = Ls > 0.f ? 1.f / Ls : 0.f;
+#pragma unroll
+            for (int i = 0; i < HD / 32; ++i)
+              outp[(rowbase + g) * HD + lane + 32 * i] = Elem<T>::from_f(o[i] * inv);
+          }
+          if (lane == 0) p.counters[cc.b * Hkv + cc.h] = 0;
+        }
+      }
+      piece_first = false;
+    }
+    if (chunk_end) {  // continue with the chunk the producer moved on to
+      if (chunk_for_consumer < 0) producer_step();  // a chunk shorter than the ring
+      c_chunk = chunk_for_consumer;
+      if (c_chunk < 0 || c_chunk >= nchunks) break;
+      cx = chunk_begin(c_chunk);
+      cend = chunk_end_x(c_chunk);
+      cc = locate(cx, pre, B, Hkv);
+      piece_first = true;
+    } else {
+      ++cx;
+      advance(cc, pre, B, Hkv);
+    }
+  }
+}
+
+template <typename T, int HD, int G, int SB>
+inline cudaError_t launch_t(const AttnParams& p, int grid, size_t smem, cudaStream_t stream) {
+  static size_t smem_set = 0;  // largest dynamic smem opted into so far
+  auto kern = decode_attn_kernel<T, HD, G, SB>;
+  if (smem > smem_set) {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    smem_set = smem;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, p);
+}
+
+template <typename T, int HD, int SB>
+inline cudaError_t launch_g(const AttnParams& p, int G, int grid, size_t smem, cudaStream_t s) {
+  switch (G) {
+    case 1: return launch_t<T, HD, 1, SB>(p, grid, smem, s);
+    case 2: return launch_t<T, HD, 2, SB>(p, grid, smem, s);
+    case 4: return launch_t<T, HD, 4, SB>(p, grid, smem, s);
+    case 8: return launch_t<T, HD, 8, SB>(p, grid, smem, s);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+}  // namespace attn_detail
+
+// Per-dtype dispatch (one translation unit each, compiled in parallel).
+cudaError_t launch_attn_bf16(const AttnParams& p, int stage_bytes, int d, int G, int grid,
+                             size_t smem, cudaStream_t s);
+cudaError_t launch_attn_f32(const AttnParams& p, int stage_bytes, int d, int G, int grid,
+                            size_t smem, cudaStream_t s);
+
+}  // namespace wm

@@ -28,6 +28,10 @@ struct AttnParams {
   float qscale;           // log2(e) / sqrt(d)
 };
 
+// Resident CTAs per SM the attention kernel is built for: 4 with 4 KB stages
+// and one query head per kv head, else 2 (GQA keeps G query rows per lane).
+constexpr int attn_ctas_per_sm(int stage_bytes, int G) { return stage_bytes == 4096 && G == 1 ? 4 : 2; }
+
 int attn_stage_slots(int stage_bytes, int dtype, int d);
 int attn_warps_per_cta();
 size_t attn_smem_bytes(int stage_bytes, int dtype, int d, int G, int B);

@@ -330,9 +330,12 @@ __global__ void __launch_bounds__(kMixThreads) mix_kernel(const MixParams p) {
 }
 
 // ---------------------------------------------------------------- epilogue
+// fp32 path: one CTA per (token, channel, branch), a warp per kv head; lane t
+// handles the RoPE pairs (i, i + HD/2) for i = t, t + 32, ...
 template <typename T, int HD>
 __global__ void __launch_bounds__(128) kv_epilogue_kernel(const MixParams p) {
-  constexpr int EPL = HD / 32;  // elements per lane; pairs (e, e + HD/2) share a lane
+  constexpr int HALF = HD / 2;
+  constexpr int NP = (HALF + 31) / 32;
   const int b = blockIdx.x, j = blockIdx.y, X = blockIdx.z;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   pdl_wait();
@@ -352,31 +355,40 @@ __global__ void __launch_bounds__(128) kv_epilogue_kernel(const MixParams p) {
   const int64_t base = (((int64_t)j * p.num_pages + pg) * p.Hkv) * p.P + (s & (p.P - 1));
   const T* qg = reinterpret_cast<const T*>(p.qk_g) + (int64_t)j * HD;
   for (int hh = warp; hh < p.Hkv; hh += 4) {
-    float y[EPL];
+    float y0[NP], y1[NP];
 #pragma unroll
-    for (int i = 0; i < EPL; ++i) y[i] = src[hh * HD + lane + 32 * i];
+    for (int t = 0; t < NP; ++t) {
+      const int i = lane + 32 * t;
+      y0[t] = i < HALF ? src[hh * HD + i] : 0.f;
+      y1[t] = i < HALF ? src[hh * HD + i + HALF] : 0.f;
+    }
     if (X == 0) {
       float ss = 0.f;
 #pragma unroll
-      for (int i = 0; i < EPL; ++i) ss = fmaf(y[i], y[i], ss);
+      for (int t = 0; t < NP; ++t) ss = fmaf(y0[t], y0[t], fmaf(y1[t], y1[t], ss));
       ss = warp_sum(ss);
       const float rr = rsqrtf(ss / (float)HD + p.eps_qk);
 #pragma unroll
-      for (int i = 0; i < EPL; ++i) y[i] = y[i] * rr * ldf(qg + lane + 32 * i);
-      // rotate-half RoPE: element e pairs with e + HD/2, both held by this lane
-#pragma unroll
-      for (int i = 0; i < EPL / 2; ++i) {
-        const int e = lane + 32 * i;
-        const float cs = p.rope_cs[((int64_t)b * (HD / 2) + e) * 2];
-        const float sn = p.rope_cs[((int64_t)b * (HD / 2) + e) * 2 + 1];
-        const float x0 = y[i], x1 = y[i + EPL / 2];
-        y[i] = x0 * cs - x1 * sn;
-        y[i + EPL / 2] = x1 * cs + x0 * sn;
+      for (int t = 0; t < NP; ++t) {
+        const int i = lane + 32 * t;
+        if (i < HALF) {
+          const float x0 = y0[t] * rr * ldf(qg + i), x1 = y1[t] * rr * ldf(qg + i + HALF);
+          const float cs = p.rope_cs[((int64_t)b * HALF + i) * 2];
+          const float sn = p.rope_cs[((int64_t)b * HALF + i) * 2 + 1];
+          y0[t] = x0 * cs - x1 * sn;  // rotate-half RoPE
+          y1[t] = x1 * cs + x0 * sn;
+        }
       }
     }
     T* dst = pool + (base + (int64_t)hh * p.P) * HD;
 #pragma unroll
-    for (int i = 0; i < EPL; ++i) dst[lane + 32 * i] = Elem<T>::from_f(y[i]);
+    for (int t = 0; t < NP; ++t) {
+      const int i = lane + 32 * t;
+      if (i < HALF) {
+        dst[i] = Elem<T>::from_f(y0[t]);
+        dst[i + HALF] = Elem<T>::from_f(y1[t]);
+      }
+    }
   }
 }
 
@@ -437,6 +449,7 @@ cudaError_t launch_all(MixParams& p, cudaStream_t s) {
   {
     dim3 grid(p.B, p.k, 2);
     if (p.d == 64) return launch_pdl(kv_epilogue_kernel<T, 64>, grid, dim3(128), 0, s, p);
+    if (p.d == 96) return launch_pdl(kv_epilogue_kernel<T, 96>, grid, dim3(128), 0, s, p);
     return launch_pdl(kv_epilogue_kernel<T, 128>, grid, dim3(128), 0, s, p);
   }
 }

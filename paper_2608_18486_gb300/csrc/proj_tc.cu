@@ -10,7 +10,9 @@
 // Shape: at decode the token count B is small (16..64) while the weights
 // are large (Hkv*d x D per channel and branch), so the weights take the MMA's
 // M side ("swap AB"): one CTA computes a 128-row tile of W^X_j against all
-// B tokens, D[row][token] in TMEM (128 lanes x N fp32 columns).  The work is
+// B tokens, D[row][token] in TMEM (128 lanes x N fp32 columns).  A projection
+// tile covers whole heads (two of d=64, one of d=96 or 128; rows past the
+// last head are computed and ignored).  The work is
 // weight-streaming bound; TMA brings 128x64 weight tiles and Nx64 token
 // tiles (128-byte swizzle) through a 4-stage mbarrier pipeline.  Warp 0 lane
 // 0 issues TMA, warp 1 lane 0 issues tcgen05.mma; all four warps drain TMEM
@@ -51,13 +53,12 @@ struct ProjTcParams {
   int32_t* status;
 };
 
-// MODE kEpiKV: grid (Hkv*d/128, k, 2) = (row tile, channel j, branch X).
+// MODE kEpiKV: grid (ceil(Hkv/hpt), k, 2) = (head tile, channel j, branch X), hpt = 128/HD.
 // MODE kEpiPartial: grid (ceil(kL/128), nsplit, 2) = (row tile, split, branch X).
 template <int HD, int MODE>
 __global__ void __launch_bounds__(kTcThreads, 1)
     proj_tc_kernel(const __grid_constant__ CUtensorMap tmW0, const __grid_constant__ CUtensorMap tmW1,
                    const __grid_constant__ CUtensorMap tmX, const ProjTcParams p) {
-  constexpr int EPL = HD / 32;
   extern __shared__ uint8_t smem_dyn[];
   __shared__ uint64_t full[kTcMaxStages], empty[kTcMaxStages], done;
   __shared__ uint32_t tmem_base;
@@ -108,7 +109,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   __syncthreads();
   tc::fence_after_sync();
   const uint32_t tmem = tmem_base;
-  const int wrow = MODE == kEpiKV ? j * p.M_item + mt * kTcM : mt * kTcM;
+  constexpr int HPT = kTcM / HD;  // whole heads per 128-row tile
+  const int wrow = MODE == kEpiKV ? j * p.M_item + mt * HPT * HD : mt * kTcM;
   const int xrow = MODE == kEpiKV ? (X * p.k + j) * p.B : X * p.B;
   const int kb0 = MODE == kEpiKV ? 0 : j * p.kb_per_split;
   const int kb1 = MODE == kEpiKV ? p.nk : min(p.nk, kb0 + p.kb_per_split);
@@ -182,47 +184,64 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     }
     return;
   }
-  // per (token, head) epilogue: keys QK-norm + RoPE, bf16 write to the cache slot
-  const int hpt = kTcM / HD;
+  // per (token, head) epilogue: keys QK-norm + RoPE, bf16 write to the cache slot.
+  // Lane t handles the RoPE pairs (i, i + HD/2) for i = t, t + 32, ...
+  constexpr int HALF = HD / 2;
+  constexpr int NP = (HALF + 31) / 32;  // pairs per lane
   const bool reporter = (mt == 0 && j == 0 && X == 0);
   __nv_bfloat16* pool = X == 0 ? p.k_pool : p.v_pool;
-  float qgv[EPL];  // QK-norm gain of channel j, the same for every item of this CTA
+  float qg0[NP], qg1[NP];  // QK-norm gain of channel j, the same for every item of this CTA
 #pragma unroll
-  for (int i = 0; i < EPL; ++i) qgv[i] = __bfloat162float(p.qk_g[(int64_t)j * HD + lane + 32 * i]);
+  for (int t = 0; t < NP; ++t) {
+    const int i = lane + 32 * t;
+    qg0[t] = i < HALF ? __bfloat162float(p.qk_g[(int64_t)j * HD + i]) : 0.f;
+    qg1[t] = i < HALF ? __bfloat162float(p.qk_g[(int64_t)j * HD + i + HALF]) : 0.f;
+  }
   const float* cs_tab = p.rope_smem_off > 0 ? rope_s : p.rope_cs;
-  for (int it = warp; it < p.B * hpt; it += kTcThreads / 32) {
-    const int n = it / hpt, hl = it % hpt;
-    const int hh = mt * hpt + hl;
+  for (int it = warp; it < p.B * HPT; it += kTcThreads / 32) {
+    const int n = it / HPT, hl = it % HPT;
+    const int hh = mt * HPT + hl;
+    if (hh >= p.Hkv) continue;
     const int s = s_slot[n], pg = s_page[n];
     if (pg < 0) {
       if (reporter && hl == 0 && lane == 0) report(p.status, WM_ERR_BOUNDS);
       continue;
     }
-    float y[EPL];
+    const float* src = T + n * kTcM + hl * HD;
+    float y0[NP], y1[NP];
 #pragma unroll
-    for (int i = 0; i < EPL; ++i) y[i] = T[n * kTcM + hl * HD + lane + 32 * i];
+    for (int t = 0; t < NP; ++t) {
+      const int i = lane + 32 * t;
+      y0[t] = i < HALF ? src[i] : 0.f;
+      y1[t] = i < HALF ? src[i + HALF] : 0.f;
+    }
     if (X == 0) {
       float ss = 0.f;
 #pragma unroll
-      for (int i = 0; i < EPL; ++i) ss = fmaf(y[i], y[i], ss);
+      for (int t = 0; t < NP; ++t) ss = fmaf(y0[t], y0[t], fmaf(y1[t], y1[t], ss));
       ss = warp_sum(ss);
       const float rr = rsqrtf(ss / (float)HD + p.eps_qk);
 #pragma unroll
-      for (int i = 0; i < EPL; ++i) y[i] = y[i] * rr * qgv[i];
-#pragma unroll
-      for (int i = 0; i < EPL / 2; ++i) {
-        const int e = lane + 32 * i;
-        const float2 csn = reinterpret_cast<const float2*>(cs_tab)[n * (HD / 2) + e];
-        const float cs = csn.x, sn = csn.y;
-        const float x0 = y[i], x1 = y[i + EPL / 2];
-        y[i] = x0 * cs - x1 * sn;
-        y[i + EPL / 2] = x1 * cs + x0 * sn;
+      for (int t = 0; t < NP; ++t) {
+        const int i = lane + 32 * t;
+        if (i < HALF) {
+          const float x0 = y0[t] * rr * qg0[t], x1 = y1[t] * rr * qg1[t];
+          const float2 csn = reinterpret_cast<const float2*>(cs_tab)[n * HALF + i];
+          y0[t] = x0 * csn.x - x1 * csn.y;  // rotate-half RoPE
+          y1[t] = x1 * csn.x + x0 * csn.y;
+        }
       }
     }
     __nv_bfloat16* dst =
         pool + ((((int64_t)j * p.num_pages + pg) * p.Hkv + hh) * p.P + (s & (p.P - 1))) * HD;
 #pragma unroll
-    for (int i = 0; i < EPL; ++i) dst[lane + 32 * i] = __float2bfloat16_rn(y[i]);
+    for (int t = 0; t < NP; ++t) {
+      const int i = lane + 32 * t;
+      if (i < HALF) {
+        dst[i] = __float2bfloat16_rn(y0[t]);
+        dst[i + HALF] = __float2bfloat16_rn(y1[t]);
+      }
+    }
   }
 }
 
@@ -308,7 +327,8 @@ cudaError_t launch_mode(dim3 grid, size_t smem, const CUtensorMap& w0, const CUt
 }  // namespace
 
 bool proj_tc_supported(const MixParams& mp) {
-  return (mp.Hkv * mp.d) % kTcM == 0 && mp.B >= 1 && mp.B <= kTcMaxTokens && encode_fn() != nullptr;
+  return (mp.d == 64 || mp.d == 96 || mp.d == 128) && mp.B >= 1 && mp.B <= kTcMaxTokens &&
+         encode_fn() != nullptr;
 }
 
 bool router_tc_supported(int B) { return B >= 1 && B <= kTcMaxTokens; }
@@ -352,7 +372,8 @@ cudaError_t launch_proj_tc(const MixParams& mp, cudaStream_t s) {
       return cudaErrorInvalidValue;
   if (!encode_kmajor(&tmX, mp.xop, (uint64_t)2 * mp.k * mp.B, mp.D, (uint32_t)p.BN))
     return cudaErrorInvalidValue;
-  dim3 grid(p.M_item / kTcM, mp.k, 2);
+  const int hpt = kTcM / mp.d;
+  dim3 grid((mp.Hkv + hpt - 1) / hpt, mp.k, 2);
   p.stages = pick_stages(p.nk, p.BN, (int64_t)grid.x * grid.y * grid.z, sm_count_cur());
   size_t smem = tc_smem(p.stages, p.BN);
   const size_t rope_bytes = (size_t)mp.B * mp.d * sizeof(float);
@@ -361,6 +382,7 @@ cudaError_t launch_proj_tc(const MixParams& mp, cudaStream_t s) {
     smem += rope_bytes;
   }
   if (mp.d == 64) return launch_mode<64, kEpiKV>(grid, smem, tmW[0], tmW[1], tmX, p, s);
+  if (mp.d == 96) return launch_mode<96, kEpiKV>(grid, smem, tmW[0], tmW[1], tmX, p, s);
   return launch_mode<128, kEpiKV>(grid, smem, tmW[0], tmW[1], tmX, p, s);
 }
 

@@ -5,6 +5,7 @@
 
 #include <mutex>
 
+#include "common.cuh"
 #include "internal.h"
 #include "wm.h"
 
@@ -59,7 +60,7 @@ AttnPlan attn_plan(const wm_config& c, int32_t B, int32_t max_pages) {
   const int64_t max_slots = (int64_t)max_pages * c.page_size;
   const double kv_bytes = (double)B * c.Hkv * max_slots * 2.0 * c.d * elem_size(c.dtype);
   pl.stage_bytes = kv_bytes < kAttnSmallLaunchBytes ? 4096 : 8192;
-  const int ctas_per_sm = pl.stage_bytes == 4096 ? 4 : 2;
+  const int ctas_per_sm = wm::attn_ctas_per_sm(pl.stage_bytes, c.Hq / c.Hkv);
   const int stage = wm::attn_stage_slots(pl.stage_bytes, c.dtype, c.d);
   const int64_t ns_max = (int64_t)B * c.Hkv * ((max_slots + stage - 1) / stage);
   const int wpc = wm::attn_warps_per_cta();
@@ -127,7 +128,7 @@ wm_status wm_config_check(const wm_config* c) {
   for (int l = 0; l < c->L; ++l)
     if (c->chan_of_layer[l] < 0 || c->chan_of_layer[l] >= c->k) return WM_ERR_INVALID_ARG;
   // shapes this library builds
-  if (c->d != 64 && c->d != 128) return WM_ERR_UNSUPPORTED;
+  if (c->d != 64 && c->d != 96 && c->d != 128) return WM_ERR_UNSUPPORTED;
   const int G = c->Hq / c->Hkv;
   if (G != 1 && G != 2 && G != 4 && G != 8) return WM_ERR_UNSUPPORTED;
   if (c->D % 8 != 0 || c->D > 4096) return WM_ERR_UNSUPPORTED;
@@ -294,6 +295,29 @@ wm_status wm_kv_mix(const wm_config* c, const wm_cache* cache, const wm_mix_weig
 }
 
 }  // extern "C"
+
+// ------------------------------------------------------------------------
+// Self-test of the bounded pipeline wait: one thread waits on an mbarrier
+// that nothing arrives on, with the same helper the kernels use, gives up
+// after limit_us microseconds and reports WM_ERR_TIMEOUT.
+namespace {
+__global__ void wait_selftest_kernel(int32_t* status, uint64_t limit_ns) {
+  __shared__ uint64_t bar;
+  if (threadIdx.x != 0) return;
+  wm::mbar_init(&bar, 1);
+  wm::fence_mbar_init();
+  if (!wm::mbar_wait(&bar, 0, limit_ns)) wm::report(status, WM_ERR_TIMEOUT);
+  // the barrier's pending arrival is never made; shared memory is released
+  // with the block
+}
+}  // namespace
+
+extern "C" wm_status wm_selftest_bounded_wait(int32_t* dev_status, uint32_t limit_us,
+                                              void* stream) {
+  if (!dev_status || limit_us == 0 || limit_us > 2000000u) return WM_ERR_INVALID_ARG;
+  wait_selftest_kernel<<<1, 32, 0, (cudaStream_t)stream>>>(dev_status, (uint64_t)limit_us * 1000ull);
+  return cudaGetLastError() == cudaSuccess ? WM_OK : WM_ERR_CUDA;
+}
 
 // ------------------------------------------------------------------------
 // Decode attention without caller-provided scratch.

@@ -40,7 +40,7 @@ def cfg(**kw):
 @pytest.mark.parametrize("field,value,code", [
     ("k", 33, W.WM_ERR_INVALID_ARG), ("k", 0, W.WM_ERR_INVALID_ARG),
     ("Hq", 33, W.WM_ERR_INVALID_ARG), ("p", 0, W.WM_ERR_INVALID_ARG),
-    ("dtype", 7, W.WM_ERR_INVALID_ARG), ("d", 96, W.WM_ERR_UNSUPPORTED),
+    ("dtype", 7, W.WM_ERR_INVALID_ARG), ("d", 80, W.WM_ERR_UNSUPPORTED),
     ("page_size", 24, W.WM_ERR_UNSUPPORTED), ("D", 8192, W.WM_ERR_UNSUPPORTED),
     ("Hq", 96, W.WM_ERR_UNSUPPORTED)])
 def test_config_check_codes(field, value, code):

@@ -1,0 +1,35 @@
+"""The paper's own model shape (Sec. 4.1): D=512, 6 query / 3 kv heads of
+d=96 (GQA groups of 2), L=16, k in {1, 8, 16} with the three router bias
+initialisations of Sec. 3.1 (top, cyclic, shifted identity).  GPU path vs
+the fp64 oracle, all layers and all tokens."""
+import pytest
+import torch
+
+from wm_synth import configs
+
+from . import _harness as H
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.mark.parametrize("name,overrides", [
+    ("paper_k8", dict()), ("paper_k16", dict()), ("paper_k1", dict()),
+    ("paper_k8", dict(dtype="f32", B=4, ctx=300, permute_pages=True, gain_std=0.1)),
+])
+def test_paper_shape_attention_and_pool(name, overrides):
+    w = configs.get(name).with_(**overrides)
+    prob, sess, dp = H.setup(w)
+    for layer in range(w.L):
+        got = H.to_f64(H.run_attn(sess, dp, layer))
+        want = H.oracle_attn_full(prob, layer)
+        assert H.rel_err(got, want) <= H.TOL[w.dtype], (layer, H.rel_err(got, want))
+    sess.kv_mix(dp.h, dp.page_table, dp.slot)
+    torch.cuda.synchronize()
+    assert sess.read_status() == 0
+    want = H.oracle_mix_tokens(prob)
+    for (b, j), (k, v) in want.items():
+        gk, gv = H.gpu_written_kv(sess, prob, b, j)
+        assert H.rel_err(gk, k) <= H.TOL[w.dtype], ("K", b, j, H.rel_err(gk, k))
+        assert H.rel_err(gv, v) <= H.TOL[w.dtype], ("V", b, j, H.rel_err(gv, v))
+    torch.cuda.synchronize()
+    torch.cuda.empty_cache()

@@ -81,6 +81,15 @@ WORKLOADS: dict[str, Workload] = {
     "long128k": Workload("long128k", L=32, k=8, D=4096, Hq=32, Hkv=32, d=128, B=8,
                          ctx=131072, page=64, dtype="bf16", chan_map="mod",
                          permute_pages=True),
+    # the paper's own model shape (Sec. 4.1): Qwen3 D=512, 6 query / 3 kv heads
+    # of dimension 96, L=16; k=16 (full cache), k=8 (half cache) and k=1.
+    # Decode batch 16 at the training length 2048 (the paper fixes no decode batch).
+    "paper_k16": Workload("paper_k16", L=16, k=16, D=512, Hq=6, Hkv=3, d=96, B=16, ctx=2048,
+                          page=16, dtype="bf16", chan_map="mod"),
+    "paper_k8": Workload("paper_k8", L=16, k=8, D=512, Hq=6, Hkv=3, d=96, B=16, ctx=2048,
+                         page=16, dtype="bf16", chan_map="mod"),
+    "paper_k1": Workload("paper_k1", L=16, k=1, D=512, Hq=6, Hkv=3, d=96, B=16, ctx=2048,
+                         page=16, dtype="bf16", chan_map="mod"),
 }
 
 

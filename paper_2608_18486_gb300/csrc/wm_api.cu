@@ -43,8 +43,9 @@ struct AttnPlan {
 
 constexpr int kAttnMaxBatch = 4096;
 // Launches reading less than this many KV bytes (upper bound from the page
-// table width) use 4 KB stages and 4 CTAs per SM (16 warps: more latency
-// hiding for short launches); larger ones use 8 KB stages and 2 CTAs per SM.
+// table width) with one query head per kv head use 4 KB stages and 4 CTAs
+// per SM (16 warps: more latency hiding for short launches); larger ones and
+// grouped-query launches (2 CTAs per SM either way) use 8 KB stages.
 constexpr double kAttnSmallLaunchBytes = 1.0e9;
 // Launches reading at least this many KV bytes hand out work dynamically:
 // chunks of the stage stream taken from an atomic counter, about
@@ -59,7 +60,7 @@ AttnPlan attn_plan(const wm_config& c, int32_t B, int32_t max_pages) {
   AttnPlan pl{};
   const int64_t max_slots = (int64_t)max_pages * c.page_size;
   const double kv_bytes = (double)B * c.Hkv * max_slots * 2.0 * c.d * elem_size(c.dtype);
-  pl.stage_bytes = kv_bytes < kAttnSmallLaunchBytes ? 4096 : 8192;
+  pl.stage_bytes = (kv_bytes < kAttnSmallLaunchBytes && c.Hq == c.Hkv) ? 4096 : 8192;
   const int ctas_per_sm = wm::attn_ctas_per_sm(pl.stage_bytes, c.Hq / c.Hkv);
   const int stage = wm::attn_stage_slots(pl.stage_bytes, c.dtype, c.d);
   const int64_t ns_max = (int64_t)B * c.Hkv * ((max_slots + stage - 1) / stage);

@@ -53,8 +53,10 @@ struct ProjTcParams {
   int32_t* status;
 };
 
-// MODE kEpiKV: grid (ceil(Hkv/hpt), k, 2) = (head tile, channel j, branch X), hpt = 128/HD.
-// MODE kEpiPartial: grid (ceil(kL/128), nsplit, 2) = (row tile, split, branch X).
+// MODE kEpiKV: grid (ceil(Hkv/hpt), k, 2*ntiles) = (head tile, channel j, branch X + 2*token
+// tile), hpt = 128/HD.
+// MODE kEpiPartial: grid (ceil(kL/128), nsplit, 2*ntiles) = (row tile, split, branch X + 2*token
+// tile).  A token tile is BN <= 256 tokens.
 template <int HD, int MODE>
 __global__ void __launch_bounds__(kTcThreads, 1)
     proj_tc_kernel(const __grid_constant__ CUtensorMap tmW0, const __grid_constant__ CUtensorMap tmW1,
@@ -64,7 +66,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   __shared__ uint32_t tmem_base;
   __shared__ int s_slot[kTcMaxTokens], s_page[kTcMaxTokens];
 
-  const int mt = blockIdx.x, j = blockIdx.y, X = blockIdx.z;
+  const int mt = blockIdx.x, j = blockIdx.y, X = blockIdx.z & 1;
+  const int n0 = (blockIdx.z >> 1) * p.BN;      // first token of this tile
+  const int nb = min(p.BN, p.B - n0);           // tokens in this tile
   const int NS = p.stages;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const CUtensorMap* tmW = X == 0 ? &tmW0 : &tmW1;
@@ -91,12 +95,13 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   float* rope_s = reinterpret_cast<float*>(base + p.rope_smem_off);  // [B][HD/2][2] or unused
   if (MODE == kEpiKV) {
     if (p.rope_smem_off > 0)
-      for (int i = threadIdx.x; i < p.B * HD; i += kTcThreads) rope_s[i] = p.rope_cs[i];
-    // destination slot and page of every token, read before the K loop
-    for (int n = threadIdx.x; n < p.B; n += kTcThreads) {
-      const int s = p.slot[n];
+      for (int i = threadIdx.x; i < nb * HD; i += kTcThreads) rope_s[i] = p.rope_cs[(int64_t)n0 * HD + i];
+    // destination slot and page of every token of the tile, read before the K loop
+    for (int n = threadIdx.x; n < nb; n += kTcThreads) {
+      const int s = p.slot[n0 + n];
       int pg = -1;
-      if (s >= 1 && s < p.max_pages * p.P) pg = p.page_table[(int64_t)n * p.max_pages + (s >> p.log2P)];
+      if (s >= 1 && s < p.max_pages * p.P)
+        pg = p.page_table[(int64_t)(n0 + n) * p.max_pages + (s >> p.log2P)];
       s_slot[n] = s;
       s_page[n] = (pg >= 0 && pg < p.num_pages) ? pg : -1;
     }
@@ -111,7 +116,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   const uint32_t tmem = tmem_base;
   constexpr int HPT = kTcM / HD;  // whole heads per 128-row tile
   const int wrow = MODE == kEpiKV ? j * p.M_item + mt * HPT * HD : mt * kTcM;
-  const int xrow = MODE == kEpiKV ? (X * p.k + j) * p.B : X * p.B;
+  const int xrow = (MODE == kEpiKV ? (X * p.k + j) * p.B : X * p.B) + n0;
   const int kb0 = MODE == kEpiKV ? 0 : j * p.kb_per_split;
   const int kb1 = MODE == kEpiKV ? p.nk : min(p.nk, kb0 + p.kb_per_split);
   const int nkb = kb1 - kb0;
@@ -176,9 +181,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 
   if (MODE == kEpiPartial) {
     // fp32 partial logits of this split: zpart[X][split][n][row]
-    float* z = p.zpart + (((int64_t)X * gridDim.y + j) * p.B) * p.M_total;
+    float* z = p.zpart + (((int64_t)X * gridDim.y + j) * p.B + n0) * p.M_total;
     const int m0 = mt * kTcM;
-    for (int i = threadIdx.x; i < p.B * kTcM; i += kTcThreads) {
+    for (int i = threadIdx.x; i < nb * kTcM; i += kTcThreads) {
       const int n = i / kTcM, r = i % kTcM;
       if (m0 + r < p.M_total) z[(int64_t)n * p.M_total + m0 + r] = T[n * kTcM + r];
     }
@@ -198,8 +203,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     qg1[t] = i < HALF ? __bfloat162float(p.qk_g[(int64_t)j * HD + i + HALF]) : 0.f;
   }
   const float* cs_tab = p.rope_smem_off > 0 ? rope_s : p.rope_cs;
-  for (int it = warp; it < p.B * HPT; it += kTcThreads / 32) {
-    const int n = it / HPT, hl = it % HPT;
+  for (int it = warp; it < nb * HPT; it += kTcThreads / 32) {
+    const int n = it / HPT, hl = it % HPT;  // n: token within the tile
     const int hh = mt * HPT + hl;
     if (hh >= p.Hkv) continue;
     const int s = s_slot[n], pg = s_page[n];
@@ -226,7 +231,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         const int i = lane + 32 * t;
         if (i < HALF) {
           const float x0 = y0[t] * rr * qg0[t], x1 = y1[t] * rr * qg1[t];
-          const float2 csn = reinterpret_cast<const float2*>(cs_tab)[n * HALF + i];
+          const float2 csn = reinterpret_cast<const float2*>(cs_tab)[(cs_tab == rope_s ? n : n0 + n) * HALF + i];
           y0[t] = x0 * csn.x - x1 * csn.y;  // rotate-half RoPE
           y1[t] = x1 * csn.x + x0 * csn.y;
         }
@@ -326,16 +331,21 @@ cudaError_t launch_mode(dim3 grid, size_t smem, const CUtensorMap& w0, const CUt
 
 }  // namespace
 
-bool proj_tc_supported(const MixParams& mp) {
-  return (mp.d == 64 || mp.d == 96 || mp.d == 128) && mp.B >= 1 && mp.B <= kTcMaxTokens &&
-         encode_fn() != nullptr;
+int token_tile(int B) {  // tokens per MMA N tile: a multiple of 16, at most 256
+  const int t = B < kTcMaxTokens ? B : kTcMaxTokens;
+  return (t + 15) / 16 * 16;
 }
 
-bool router_tc_supported(int B) { return B >= 1 && B <= kTcMaxTokens; }
+bool proj_tc_supported(const MixParams& mp) {
+  return (mp.d == 64 || mp.d == 96 || mp.d == 128) && mp.B >= 1 && encode_fn() != nullptr;
+}
+
+bool router_tc_supported(int B) { return B >= 1; }
 
 int router_tc_splits(int k, int L, int Lp, int D, int B, int sms) {
   const int nk = (Lp * D + kTcBK - 1) / kTcBK;
-  const int tiles = 2 * ((k * L + kTcM - 1) / kTcM);
+  const int ntiles = (B + token_tile(B) - 1) / token_tile(B);
+  const int tiles = 2 * ((k * L + kTcM - 1) / kTcM) * ntiles;
   int ns = (sms + tiles - 1) / tiles;
   const int max_ns = nk / 8 > 1 ? nk / 8 : 1;  // at least 8 k-blocks per split
   ns = ns < 1 ? 1 : (ns > max_ns ? max_ns : ns);
@@ -351,7 +361,7 @@ cudaError_t launch_proj_tc(const MixParams& mp, cudaStream_t s) {
   p.Hkv = mp.Hkv;
   p.D = mp.D;
   p.M_item = mp.Hkv * mp.d;
-  p.BN = (mp.B + 15) / 16 * 16;
+  p.BN = token_tile(mp.B);
   p.nk = (mp.D + kTcBK - 1) / kTcBK;
   p.P = mp.P;
   p.log2P = mp.log2P;
@@ -373,10 +383,11 @@ cudaError_t launch_proj_tc(const MixParams& mp, cudaStream_t s) {
   if (!encode_kmajor(&tmX, mp.xop, (uint64_t)2 * mp.k * mp.B, mp.D, (uint32_t)p.BN))
     return cudaErrorInvalidValue;
   const int hpt = kTcM / mp.d;
-  dim3 grid((mp.Hkv + hpt - 1) / hpt, mp.k, 2);
+  const int ntiles = (mp.B + p.BN - 1) / p.BN;
+  dim3 grid((mp.Hkv + hpt - 1) / hpt, mp.k, 2 * ntiles);
   p.stages = pick_stages(p.nk, p.BN, (int64_t)grid.x * grid.y * grid.z, sm_count_cur());
   size_t smem = tc_smem(p.stages, p.BN);
-  const size_t rope_bytes = (size_t)mp.B * mp.d * sizeof(float);
+  const size_t rope_bytes = (size_t)p.BN * mp.d * sizeof(float);
   if (smem + rope_bytes <= 200 * 1024) {
     p.rope_smem_off = (int32_t)(smem - 1024);  // offset from the 1 KB-aligned base
     smem += rope_bytes;
@@ -393,7 +404,7 @@ cudaError_t launch_router_tc(const MixParams& mp, cudaStream_t s) {
   p.k = mp.k;
   p.B = mp.B;
   p.D = K;
-  p.BN = (mp.B + 15) / 16 * 16;
+  p.BN = token_tile(mp.B);
   p.nk = (K + kTcBK - 1) / kTcBK;
   p.kb_per_split = (p.nk + mp.nsplit_r - 1) / mp.nsplit_r;
   p.M_total = kL;
@@ -405,7 +416,7 @@ cudaError_t launch_router_tc(const MixParams& mp, cudaStream_t s) {
     if (!encode_kmajor(&tmW[X], mp.Wr[X], (uint64_t)kL, K, kTcM)) return cudaErrorInvalidValue;
   if (!encode_kmajor(&tmX, mp.xi, (uint64_t)2 * mp.B, K, (uint32_t)p.BN))
     return cudaErrorInvalidValue;
-  dim3 grid((kL + kTcM - 1) / kTcM, mp.nsplit_r, 2);
+  dim3 grid((kL + kTcM - 1) / kTcM, mp.nsplit_r, 2 * ((mp.B + p.BN - 1) / p.BN));
   p.stages = pick_stages(p.kb_per_split, p.BN, (int64_t)grid.x * grid.y * grid.z, sm_count_cur());
   const size_t smem = tc_smem(p.stages, p.BN);
   return launch_mode<64, kEpiPartial>(grid, smem, tmW[0], tmW[1], tmX, p, s);

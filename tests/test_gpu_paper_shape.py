@@ -33,3 +33,25 @@ def test_paper_shape_attention_and_pool(name, overrides):
         assert H.rel_err(gv, v) <= H.TOL[w.dtype], ("V", b, j, H.rel_err(gv, v))
     torch.cuda.synchronize()
     torch.cuda.empty_cache()
+
+
+@pytest.mark.parametrize("B,g", [(300, 8), (600, 16)])
+def test_batched_pool_over_several_token_tiles(B, g):
+    """The pool for a prefill-sized batch (Sec. 3.3: a Gauss-Seidel group of
+    strided positions i = q (mod g) across sequences): more tokens than one
+    tensor-core token tile (256), written to strided slots."""
+    w = configs.get("paper_k8").with_(B=B, ctx=8 * g + 64, permute_pages=True)
+    # token b sits at position q + g*t of its row: strided slots, distinct per row
+    lens = [1 + (b % g) + g * ((b // g) % 8) for b in range(B)]
+    prob, sess, dp = H.setup(w, seq_lens=lens, fill_pools=False)
+    sess.kv_mix(dp.h, dp.page_table, dp.slot)
+    torch.cuda.synchronize()
+    assert sess.read_status() == 0
+    tokens = [0, 1, 255, 256, 257, B - 1] + ([511, 512] if B > 512 else [])
+    want = H.oracle_mix_tokens(prob, tokens=tokens, chans=(0, 3, 7))
+    for (b, j), (k, v) in want.items():
+        gk, gv = H.gpu_written_kv(sess, prob, b, j)
+        assert H.rel_err(gk, k) <= H.TOL[w.dtype], ("K", b, j, H.rel_err(gk, k))
+        assert H.rel_err(gv, v) <= H.TOL[w.dtype], ("V", b, j, H.rel_err(gv, v))
+    torch.cuda.synchronize()
+    torch.cuda.empty_cache()

@@ -93,19 +93,6 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   asm volatile("griddepcontrol.wait;" ::: "memory");
   float* rope_s = reinterpret_cast<float*>(base + p.rope_smem_off);  // [B][HD/2][2] or unused
-  if (MODE == kEpiKV) {
-    if (p.rope_smem_off > 0)
-      for (int i = threadIdx.x; i < nb * HD; i += kTcThreads) rope_s[i] = p.rope_cs[(int64_t)n0 * HD + i];
-    // destination slot and page of every token of the tile, read before the K loop
-    for (int n = threadIdx.x; n < nb; n += kTcThreads) {
-      const int s = p.slot[n0 + n];
-      int pg = -1;
-      if (s >= 1 && s < p.max_pages * p.P)
-        pg = p.page_table[(int64_t)(n0 + n) * p.max_pages + (s >> p.log2P)];
-      s_slot[n] = s;
-      s_page[n] = (pg >= 0 && pg < p.num_pages) ? pg : -1;
-    }
-  }
   if (warp == 0) {
     tc::tmem_alloc(&tmem_base, p.tmem_cols);
     tc::tmem_relinquish();
@@ -132,6 +119,20 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       mbar_arrive_expect_tx(&full[s], a_bytes + b_bytes);
       tc::tma_load_2d(As + s * a_bytes, tmW, (kb0 + kb) * kTcBK, wrow, &full[s]);
       tc::tma_load_2d(Bs + s * b_bytes, &tmX, (kb0 + kb) * kTcBK, xrow, &full[s]);
+    }
+  } else if (MODE == kEpiKV && warp >= 2) {
+    // meanwhile warps 2-3 fetch what the epilogue needs: the RoPE table of the
+    // tile's tokens and each token's destination slot and page
+    const int t2 = threadIdx.x - 64;
+    if (p.rope_smem_off > 0)
+      for (int i = t2; i < nb * HD; i += 64) rope_s[i] = p.rope_cs[(int64_t)n0 * HD + i];
+    for (int n = t2; n < nb; n += 64) {
+      const int s = p.slot[n0 + n];
+      int pg = -1;
+      if (s >= 1 && s < p.max_pages * p.P)
+        pg = p.page_table[(int64_t)(n0 + n) * p.max_pages + (s >> p.log2P)];
+      s_slot[n] = s;
+      s_page[n] = (pg >= 0 && pg < p.num_pages) ? pg : -1;
     }
   } else if (warp == 1 && lane == 0) {
     // MMA issuer: 4 MMAs of K = 16 per stage

@@ -553,42 +553,43 @@ __global__ void __launch_bounds__(kThreads, attn_ctas_per_sm(SB, G)) decode_attn
         if (last) {
           __threadfence();
           // merge the pieces of chunks g_first .. g_last (side 1 of the first
-          // chunk, side 0 of the others), up to 32 pieces per round, one per lane
+          // chunk, side 0 of the others) in batches of 4-8: every load of a batch
+          // (each piece's max, sum and d-vector) is issued before any is used
+          constexpr int MB = HD >= 96 ? 4 : 8;
           const int np = (int)(g_last - g_first + 1);
           for (int g = 0; g < G; ++g) {
             float M = -INFINITY, Ls = 0.f;
             float o[HD / 32];
 #pragma unroll
             for (int i = 0; i < HD / 32; ++i) o[i] = 0.f;
-            for (int r0 = 0; r0 < np; r0 += 32) {
-              const int nr = min(32, np - r0);
-              float mq = -INFINITY, lq = 0.f;
-              if (lane < nr) {
-                const int64_t q = g_first + r0 + lane;
-                const float* pm = p.part_ml + ((int64_t)(q == g_first ? 1 : 0) * p.max_chunks + q) * G * 2 + 2 * g;
-                mq = __ldcg(pm);
-                lq = __ldcg(pm + 1);
+            for (int r0 = 0; r0 < np; r0 += MB) {
+              float mq[MB], lq[MB], ov[MB][HD / 32];
+#pragma unroll
+              for (int jb = 0; jb < MB; ++jb) {
+                const int64_t q = g_first + r0 + jb;
+                const bool in = r0 + jb < np;
+                const int64_t slot = ((int64_t)(q == g_first ? 1 : 0) * p.max_chunks + q) * G + g;
+                mq[jb] = in ? __ldcg(p.part_ml + slot * 2) : -INFINITY;
+                lq[jb] = in ? __ldcg(p.part_ml + slot * 2 + 1) : 0.f;
+#pragma unroll
+                for (int i = 0; i < HD / 32; ++i)
+                  ov[jb][i] = in ? __ldcg(p.part_o + slot * HD + lane + 32 * i) : 0.f;
               }
-              float Mr = mq;
+              float Mn = M;
 #pragma unroll
-              for (int o2 = 16; o2 > 0; o2 >>= 1) Mr = fmaxf(Mr, __shfl_xor_sync(FULLMASK, Mr, o2));
-              const float Mn = fmaxf(M, Mr);
+              for (int jb = 0; jb < MB; ++jb) Mn = fmaxf(Mn, mq[jb]);
               if (Mn == -INFINITY) continue;
-              const float rescale = exp2f(M - Mn);  // 0 on the first round
-              const float w = (mq == -INFINITY) ? 0.f : exp2f(mq - Mn);
-              float lw = w * lq;
-#pragma unroll
-              for (int o2 = 16; o2 > 0; o2 >>= 1) lw += __shfl_xor_sync(FULLMASK, lw, o2);
-              Ls = Ls * rescale + lw;
+              const float rescale = exp2f(M - Mn);  // 0 on the first batch
+              Ls *= rescale;
 #pragma unroll
               for (int i = 0; i < HD / 32; ++i) o[i] *= rescale;
-#pragma unroll 4
-              for (int j = 0; j < nr; ++j) {
-                const float wj = __shfl_sync(FULLMASK, w, j);
-                const int64_t q = g_first + r0 + j;
-                const float* po = p.part_o + (((int64_t)(q == g_first ? 1 : 0) * p.max_chunks + q) * G + g) * HD;
 #pragma unroll
-                for (int i = 0; i < HD / 32; ++i) o[i] = fmaf(wj, __ldcg(po + lane + 32 * i), o[i]);
+              for (int jb = 0; jb < MB; ++jb) {
+                if (mq[jb] == -INFINITY) continue;
+                const float w = exp2f(mq[jb] - Mn);
+                Ls = fmaf(w, lq[jb], Ls);
+#pragma unroll
+                for (int i = 0; i < HD / 32; ++i) o[i] = fmaf(w, ov[jb][i], o[i]);
               }
               M = Mn;
             }

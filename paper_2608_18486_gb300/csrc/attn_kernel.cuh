@@ -23,7 +23,10 @@
 //  * Merge.  A piece of a unit that lies inside one chunk is written straight
 //    to the output.  Only units that cross a chunk boundary leave partials
 //    (at most two per chunk: its first and its last piece); the last warp to
-//    finish such a unit (atomic ticket, no waiting) merges them.
+//    finish such a unit (atomic ticket, no waiting) merges them.  When that
+//    warp has no stage left in flight, its idle ring receives the unit's
+//    partial records with bulk copies (one round trip for up to a ring's
+//    worth), and the merge reads them from shared memory.
 #include <math.h>
 
 #include "common.cuh"
@@ -215,6 +218,14 @@ __global__ void __launch_bounds__(kThreads, attn_ctas_per_sm(SB, G)) decode_attn
   constexpr int STAGE_SLOTS = SH::STAGE_SLOTS, STAGE_ELEMS = SH::STAGE_ELEMS;
   constexpr uint32_t KV_BYTES = STAGE_ELEMS * sizeof(T);
   constexpr uint32_t Q_BYTES = G * HD * sizeof(T);
+  constexpr int REC = attn_part_rec(G, HD);                        // floats per partial record
+  constexpr int RING_RECS = (int)(kWStages * 2 * KV_BYTES / (REC * sizeof(float)));
+  static_assert(RING_RECS >= 1 && (REC * sizeof(float)) % 16 == 0, "partial records");
+  // Partial merges take pieces in batches of MB (every load of a batch issued
+  // before any is used); both merge paths run the same batches in the same
+  // order, so the result does not depend on which path a warp takes.
+  constexpr int MB = (HD >= 96 ? 4 : 8) < RING_RECS ? (HD >= 96 ? 4 : 8) : RING_RECS;
+  constexpr int ROUND = RING_RECS / MB * MB;  // records per bulk round: whole batches
   constexpr unsigned FULLMASK = 0xFFFFFFFFu;
 
   extern __shared__ __align__(128) unsigned char smem_raw[];
@@ -350,14 +361,14 @@ __global__ void __launch_bounds__(kThreads, attn_ctas_per_sm(SB, G)) decode_attn
 
   // ---- producer: walks its chunks stage by stage, kWStages ahead of the consumer
   int64_t p_chunk = gw;
-  int64_t px = chunk_begin(p_chunk), pend = chunk_end_x(p_chunk);
+  int64_t px = chunk_begin(p_chunk), pend = chunk_end_x(p_chunk), pbeg = px;
   int64_t chunk_for_consumer = -1;              // the producer's chunk after a switch
   bool p_done = false;
   Cursor pc = locate(px, pre, B, Hkv);
   uint32_t pseq = 0;                            // stages issued
   auto issue = [&]() {
     const int buf = (int)(pseq % kWStages);
-    const bool first = (px == chunk_begin(p_chunk)) || pc.st == 0;
+    const bool first = (px == pbeg) || pc.st == 0;
     const int S = lens[pc.b];
     const int s_begin = pc.st * STAGE_SLOTS;
     const T* kb = reinterpret_cast<const T*>(p.k_pool) + (int64_t)pc.h * p.P * HD;
@@ -424,6 +435,7 @@ __global__ void __launch_bounds__(kThreads, attn_ctas_per_sm(SB, G)) decode_attn
       }
       px = chunk_begin(p_chunk);
       pend = chunk_end_x(p_chunk);
+      pbeg = px;
       pc = locate(px, pre, B, Hkv);
       grab_issue();
     }
@@ -444,7 +456,7 @@ __global__ void __launch_bounds__(kThreads, attn_ctas_per_sm(SB, G)) decode_attn
   const int log2P_in_stage = p.P >= STAGE_SLOTS ? 30 : p.log2P;  // stage page index = slot >> this
   const uint64_t all_pages = p.P >= STAGE_SLOTS ? 1ull : ((1ull << (STAGE_SLOTS >> p.log2P)) - 1ull);
   int64_t c_chunk = gw;
-  int64_t cx = chunk_begin(c_chunk), cend = chunk_end_x(c_chunk);
+  int64_t cx = chunk_begin(c_chunk), cend = chunk_end_x(c_chunk), cbeg = cx;
   Cursor cc = locate(cx, pre, B, Hkv);
   bool piece_first = true;  // the current piece starts at its chunk's first stage
   float2 q2[G][E2];
@@ -464,7 +476,7 @@ __global__ void __launch_bounds__(kThreads, attn_ctas_per_sm(SB, G)) decode_attn
       __syncwarp();
       return;
     }
-    if (cx == chunk_begin(c_chunk) || cc.st == 0) {
+    if (cx == cbeg || cc.st == 0) {
       const T* qs = myq + buf * G * HD;
 #pragma unroll
       for (int g = 0; g < G; ++g) {
@@ -522,8 +534,8 @@ __global__ void __launch_bounds__(kThreads, attn_ctas_per_sm(SB, G)) decode_attn
         // partial of this piece: its chunk's first piece -> side 0, last piece -> side 1
         for (int side = 0; side < 2; ++side) {
           if ((side == 0 && !piece_first) || (side == 1 && !chunk_end)) continue;
-          float* po = p.part_o + ((int64_t)side * p.max_chunks + c_chunk) * G * HD;
-          float* pm = p.part_ml + ((int64_t)side * p.max_chunks + c_chunk) * G * 2;
+          float* po = p.part + ((int64_t)side * p.max_chunks + c_chunk) * REC;
+          float* pm = po + G * HD;
           if (lane_slot == 0) {
 #pragma unroll
             for (int g = 0; g < G; ++g)
@@ -552,51 +564,132 @@ __global__ void __launch_bounds__(kThreads, attn_ctas_per_sm(SB, G)) decode_attn
         last = __shfl_sync(FULLMASK, last, 0);
         if (last) {
           __threadfence();
-          // merge the pieces of chunks g_first .. g_last (side 1 of the first
-          // chunk, side 0 of the others) in batches of 4-8: every load of a batch
-          // (each piece's max, sum and d-vector) is issued before any is used
-          constexpr int MB = HD >= 96 ? 4 : 8;
+          // merge the pieces of chunks g_first .. g_last: side 1 of the first
+          // chunk, then side 0 of the others (consecutive records)
           const int np = (int)(g_last - g_first + 1);
-          for (int g = 0; g < G; ++g) {
-            float M = -INFINITY, Ls = 0.f;
-            float o[HD / 32];
+          const float* rec1 = p.part + (int64_t)(p.max_chunks + g_first) * REC;
+          const float* rec0 = p.part + (int64_t)(g_first + 1) * REC;
+          if (p_done && seq + 1 == pseq) {
+            // no stage in flight: the ring takes ROUND records per round
+            float* rs = reinterpret_cast<float*>(myring);
+            float M[G], Ls[G], o[G][HD / 32];
 #pragma unroll
-            for (int i = 0; i < HD / 32; ++i) o[i] = 0.f;
-            for (int r0 = 0; r0 < np; r0 += MB) {
-              float mq[MB], lq[MB], ov[MB][HD / 32];
+            for (int g = 0; g < G; ++g) {
+              M[g] = -INFINITY;
+              Ls[g] = 0.f;
 #pragma unroll
-              for (int jb = 0; jb < MB; ++jb) {
-                const int64_t q = g_first + r0 + jb;
-                const bool in = r0 + jb < np;
-                const int64_t slot = ((int64_t)(q == g_first ? 1 : 0) * p.max_chunks + q) * G + g;
-                mq[jb] = in ? __ldcg(p.part_ml + slot * 2) : -INFINITY;
-                lq[jb] = in ? __ldcg(p.part_ml + slot * 2 + 1) : 0.f;
+              for (int i = 0; i < HD / 32; ++i) o[g][i] = 0.f;
+            }
+            fence_proxy_async_global();
+            fence_proxy_async_shared();
+            bool landed = true;
+            for (int r0 = 0; r0 < np; r0 += ROUND) {
+              const int n = min(ROUND, np - r0);
+              constexpr uint32_t RB = REC * sizeof(float);
+              if (lane == 0) {
+                mbar_arrive_expect_tx(&qbars[warp], (uint32_t)n * RB);
+                if (r0 == 0) {
+                  bulk_g2s(rs, rec1, RB, &qbars[warp], policy);
+                  if (n > 1) bulk_g2s(rs + REC, rec0, (uint32_t)(n - 1) * RB, &qbars[warp], policy);
+                } else {
+                  bulk_g2s(rs, rec0 + (int64_t)(r0 - 1) * REC, (uint32_t)n * RB, &qbars[warp], policy);
+                }
+              }
+              // qbars completed phase 0 with the first query; round r is phase r + 1
+              const uint32_t parity = (uint32_t)(r0 / ROUND + 1) & 1u;
+              landed = mbar_wait(&qbars[warp], parity);
+              if (__any_sync(FULLMASK, !landed)) {
+                if (lane == 0) {
+                  report(p.status, WM_ERR_TIMEOUT);
+                  mbar_wait(&qbars[warp], parity);
+                }
+                landed = false;
+                break;
+              }
+#pragma unroll
+              for (int g = 0; g < G; ++g) {
+                for (int b0 = 0; b0 < n; b0 += MB) {
+                  float mq[MB], lq[MB];
+#pragma unroll
+                  for (int jb = 0; jb < MB; ++jb) {
+                    const bool in = b0 + jb < n;
+                    mq[jb] = in ? rs[(b0 + jb) * REC + G * HD + 2 * g] : -INFINITY;
+                    lq[jb] = in ? rs[(b0 + jb) * REC + G * HD + 2 * g + 1] : 0.f;
+                  }
+                  float Mn = M[g];
+#pragma unroll
+                  for (int jb = 0; jb < MB; ++jb) Mn = fmaxf(Mn, mq[jb]);
+                  if (Mn == -INFINITY) continue;
+                  const float rescale = exp2f(M[g] - Mn);  // 0 on the first batch
+                  Ls[g] *= rescale;
+#pragma unroll
+                  for (int i = 0; i < HD / 32; ++i) o[g][i] *= rescale;
+#pragma unroll
+                  for (int jb = 0; jb < MB; ++jb) {
+                    if (mq[jb] == -INFINITY) continue;
+                    const float w = exp2f(mq[jb] - Mn);
+                    Ls[g] = fmaf(w, lq[jb], Ls[g]);
+                    const float* rj = rs + (b0 + jb) * REC + g * HD + lane;
+#pragma unroll
+                    for (int i = 0; i < HD / 32; ++i) o[g][i] = fmaf(w, rj[32 * i], o[g][i]);
+                  }
+                  M[g] = Mn;
+                }
+              }
+              __syncwarp();  // every lane is done with the ring before the next round
+            }
+            if (landed) {
+#pragma unroll
+              for (int g = 0; g < G; ++g) {
+                const float inv = Ls[g] > 0.f ? 1.f / Ls[g] : 0.f;
 #pragma unroll
                 for (int i = 0; i < HD / 32; ++i)
-                  ov[jb][i] = in ? __ldcg(p.part_o + slot * HD + lane + 32 * i) : 0.f;
+                  outp[(rowbase + g) * HD + lane + 32 * i] = Elem<T>::from_f(o[g][i] * inv);
               }
-              float Mn = M;
-#pragma unroll
-              for (int jb = 0; jb < MB; ++jb) Mn = fmaxf(Mn, mq[jb]);
-              if (Mn == -INFINITY) continue;
-              const float rescale = exp2f(M - Mn);  // 0 on the first batch
-              Ls *= rescale;
-#pragma unroll
-              for (int i = 0; i < HD / 32; ++i) o[i] *= rescale;
-#pragma unroll
-              for (int jb = 0; jb < MB; ++jb) {
-                if (mq[jb] == -INFINITY) continue;
-                const float w = exp2f(mq[jb] - Mn);
-                Ls = fmaf(w, lq[jb], Ls);
-#pragma unroll
-                for (int i = 0; i < HD / 32; ++i) o[i] = fmaf(w, ov[jb][i], o[i]);
-              }
-              M = Mn;
             }
-            const float inv = Ls > 0.f ? 1.f / Ls : 0.f;
+          } else {
+            // stages in flight: the same batches, straight from global memory
+            for (int g = 0; g < G; ++g) {
+              float M = -INFINITY, Ls = 0.f;
+              float o[HD / 32];
 #pragma unroll
-            for (int i = 0; i < HD / 32; ++i)
-              outp[(rowbase + g) * HD + lane + 32 * i] = Elem<T>::from_f(o[i] * inv);
+              for (int i = 0; i < HD / 32; ++i) o[i] = 0.f;
+              for (int r0 = 0; r0 < np; r0 += MB) {
+                float mq[MB], lq[MB], ov[MB][HD / 32];
+#pragma unroll
+                for (int jb = 0; jb < MB; ++jb) {
+                  const int j = r0 + jb;
+                  const bool in = j < np;
+                  const float* rj = j == 0 ? rec1 : rec0 + (int64_t)(j - 1) * REC;
+                  mq[jb] = in ? __ldcg(rj + G * HD + 2 * g) : -INFINITY;
+                  lq[jb] = in ? __ldcg(rj + G * HD + 2 * g + 1) : 0.f;
+#pragma unroll
+                  for (int i = 0; i < HD / 32; ++i)
+                    ov[jb][i] = in ? __ldcg(rj + g * HD + lane + 32 * i) : 0.f;
+                }
+                float Mn = M;
+#pragma unroll
+                for (int jb = 0; jb < MB; ++jb) Mn = fmaxf(Mn, mq[jb]);
+                if (Mn == -INFINITY) continue;
+                const float rescale = exp2f(M - Mn);  // 0 on the first batch
+                Ls *= rescale;
+#pragma unroll
+                for (int i = 0; i < HD / 32; ++i) o[i] *= rescale;
+#pragma unroll
+                for (int jb = 0; jb < MB; ++jb) {
+                  if (mq[jb] == -INFINITY) continue;
+                  const float w = exp2f(mq[jb] - Mn);
+                  Ls = fmaf(w, lq[jb], Ls);
+#pragma unroll
+                  for (int i = 0; i < HD / 32; ++i) o[i] = fmaf(w, ov[jb][i], o[i]);
+                }
+                M = Mn;
+              }
+              const float inv = Ls > 0.f ? 1.f / Ls : 0.f;
+#pragma unroll
+              for (int i = 0; i < HD / 32; ++i)
+                outp[(rowbase + g) * HD + lane + 32 * i] = Elem<T>::from_f(o[i] * inv);
+            }
           }
           if (lane == 0) p.counters[cc.b * Hkv + cc.h] = 0;
         }
@@ -609,6 +702,7 @@ __global__ void __launch_bounds__(kThreads, attn_ctas_per_sm(SB, G)) decode_attn
       if (c_chunk < 0 || c_chunk >= nchunks) break;
       cx = chunk_begin(c_chunk);
       cend = chunk_end_x(c_chunk);
+      cbeg = cx;
       cc = locate(cx, pre, B, Hkv);
       piece_first = true;
     } else {

@@ -16,8 +16,9 @@ struct AttnParams {
   void* out;              // [B][Hq][d]
   const int32_t* page_table;
   const int32_t* seq_lens;
-  float* part_o;          // [2][max_chunks][G][d]: first / last piece partial of each chunk
-  float* part_ml;         // [2][max_chunks][G][2]: (max, sum) in log2 units
+  float* part;            // [2][max_chunks] records of attn_part_rec(G, d) floats: the
+                          // first / last piece partial of each chunk ([G][d] unnormalised
+                          // outputs, then (max, sum) per query head in log2 units)
   int32_t* counters;      // [B*Hkv] arrival tickets + 1 chunk counter, zero between launches
   int32_t* status;
   int64_t page_stride;    // elements between consecutive physical pages
@@ -31,6 +32,10 @@ struct AttnParams {
 // Resident CTAs per SM the attention kernel is built for: 4 with 4 KB stages
 // and one query head per kv head, else 2 (GQA keeps G query rows per lane).
 constexpr int attn_ctas_per_sm(int stage_bytes, int G) { return stage_bytes == 4096 && G == 1 ? 4 : 2; }
+
+// Floats per partial record: G*d outputs, then (max, sum) per head, padded to
+// 16 bytes so that consecutive records can be moved with one bulk copy.
+constexpr int attn_part_rec(int G, int d) { return G * d + (2 * G > 4 ? 2 * G : 4); }
 
 int attn_stage_slots(int stage_bytes, int dtype, int d);
 int attn_warps_per_cta();

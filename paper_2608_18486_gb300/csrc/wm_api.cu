@@ -38,7 +38,7 @@ bool aligned(const void* p, size_t a) { return ((uintptr_t)p % a) == 0; }
 // Persistent grid of one attention launch and its workspace layout.
 struct AttnPlan {
   int stage_bytes, grid, nwarps, chunk_stages, max_chunks;
-  size_t off_part_o, off_part_ml, off_counters, total;
+  size_t off_part, off_counters, total;
 };
 
 constexpr int kAttnMaxBatch = 4096;
@@ -84,10 +84,8 @@ AttnPlan attn_plan(const wm_config& c, int32_t B, int32_t max_pages) {
   }
   const int G = c.Hq / c.Hkv;
   size_t off = 0;
-  pl.off_part_o = off;
-  off += align256(sizeof(float) * 2 * (size_t)pl.max_chunks * G * c.d);
-  pl.off_part_ml = off;
-  off += align256(sizeof(float) * 2 * (size_t)pl.max_chunks * G * 2);
+  pl.off_part = off;
+  off += align256(sizeof(float) * 2 * (size_t)pl.max_chunks * wm::attn_part_rec(G, c.d));
   pl.off_counters = off;
   off += align256(sizeof(int32_t) * ((size_t)B * c.Hkv + 1));
   pl.total = off;
@@ -204,8 +202,7 @@ wm_status wm_decode_attn_flags(const wm_config* c, const wm_cache* cache, int32_
   p.out = out;
   p.page_table = page_table;
   p.seq_lens = seq_lens;
-  p.part_o = (float*)((char*)workspace + pl.off_part_o);
-  p.part_ml = (float*)((char*)workspace + pl.off_part_ml);
+  p.part = (float*)((char*)workspace + pl.off_part);
   p.counters = (int32_t*)((char*)workspace + pl.off_counters);
   p.status = dev_status;
   p.page_stride = (int64_t)c->Hkv * c->page_size * c->d;

@@ -53,12 +53,31 @@ def test_noalloc_matches_workspace_entry_point_on_two_calls(name, overrides):
             assert err <= H.TOL[w.dtype], (layer, err)
 
 
+# the size of the library's fixed scratch array (include/wm.h)
+NOALLOC_SCRATCH_BYTES = 8 << 20
+
+
 def test_noalloc_rejects_launches_larger_than_its_scratch():
-    # 4096 sequences x 8 query heads per kv head need more than the fixed array
+    # 4096 sequences x 8 query heads per kv head over 2 pages each: the
+    # partial records alone need far more than the fixed array
     w = configs.get("large").with_(B=4096, Hq=256, Hkv=32)
     cfg = H.config_of(w)
+    max_pages = 2
+    assert W.wm_decode_attn_workspace(cfg, w.B, max_pages) > 2 * NOALLOC_SCRATCH_BYTES
+    # Real buffers that make the call a valid launch (one cache page, every
+    # sequence one slot long on page 0), so that a wrong answer of the size
+    # check shows up as a failed assertion and never as a read of memory
+    # the call does not own.
+    dev = torch.device("cuda", 0)
     nbytes = W.wm_cache_bytes(cfg, 1)
-    cache = W.wm_cache_alloc(cfg, 1 << 40, nbytes, 1)  # a layout only; never touched
-    fake = 1 << 41
-    rc = W.wm_decode_attn_noalloc(cfg, cache, 0, fake, fake, fake, w.B, 1, fake, None, None)
+    cache_buf = torch.zeros(nbytes, dtype=torch.uint8, device=dev)
+    cache = W.wm_cache_alloc(cfg, cache_buf, nbytes, 1)
+    q = torch.zeros((w.B, w.Hq, w.d), dtype=torch.bfloat16, device=dev)
+    out = torch.empty_like(q)
+    page_table = torch.zeros((w.B, max_pages), dtype=torch.int32, device=dev)
+    seq_lens = torch.ones(w.B, dtype=torch.int32, device=dev)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    rc = W.wm_decode_attn_noalloc(cfg, cache, 0, q, page_table, seq_lens, w.B, max_pages, out,
+                                  status, None)
+    torch.cuda.synchronize()
     assert rc == W.WM_ERR_UNSUPPORTED

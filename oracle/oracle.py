@@ -53,6 +53,10 @@ def lib():
         L.orc_decode_attn.argtypes = [ctypes.c_int] * 8 + [_vp, _vp, _i32p, _i32p, _vp,
                                                            ctypes.c_int, _i32p, _dp, _i64p,
                                                            ctypes.c_int]
+        L.orc_prefill_attn.restype = ctypes.c_int
+        L.orc_prefill_attn.argtypes = [ctypes.c_int] * 8 + [_vp, _vp, _i32p, _i32p, ctypes.c_int,
+                                                            _vp, ctypes.c_int, _i32p, _dp, _i64p,
+                                                            ctypes.c_int]
         _lib = L
     return _lib
 
@@ -171,4 +175,38 @@ def decode_attn(q, k_pool, v_pool, page_table, seq_lens, *, chan, Hq, Hkv, d, P,
         raise IndexError(f"oracle decode_attn: error {rc} (page id or length out of range)")
     if full:
         out = out.reshape(B, Hq, d)
+    return (out, int(macs[0])) if return_macs else out
+
+
+def prefill_attn(q, k_pool, v_pool, page_table, pos, *, chan, Hq, Hkv, d, P, units=None,
+                 nthreads=1, return_macs=False):
+    """Sec. 3.1 Step 3 causal attention with the dummy offset of Sec. 3.2, for
+    query rows at given token positions (prefill; Jacobi / Gauss-Seidel passes
+    of Sec. 3.3).  Row r of sequence b is the query of the token at position
+    ``pos[b][r]`` and reads slots 0 .. pos of channel ``chan``.
+
+    ``q`` is [B][Tq][Hq][d]; ``k_pool``/``v_pool`` are [kch][num_pages][Hkv][P][d].
+    ``units`` lists (b, r, hq) triples (default: all).  Returns out[nunits][d]
+    (or [B][Tq][Hq][d] when ``units`` is None)."""
+    q = _c(q)
+    k_pool, v_pool = _c(k_pool), _c(v_pool)
+    pt = _c(page_table, np.int32)
+    ps = _c(pos, np.int32)
+    B, Tq = q.shape[0], q.shape[1]
+    num_pages = k_pool.shape[1]
+    full = units is None
+    if full:
+        units = [(b, r, hq) for b in range(B) for r in range(Tq) for hq in range(Hq)]
+    u = _c(np.asarray(units, dtype=np.int32).reshape(-1, 3))
+    out = np.empty((u.shape[0], d))
+    macs = np.zeros(1, dtype=np.int64)
+    rc = lib().orc_prefill_attn(Hq, Hkv, d, P, num_pages, pt.shape[1], chan, _dtcode(q),
+                                _ptr(k_pool), _ptr(v_pool), pt.ctypes.data_as(_i32p),
+                                ps.ctypes.data_as(_i32p), Tq, _ptr(q), u.shape[0],
+                                u.ctypes.data_as(_i32p), _dptr(out), macs.ctypes.data_as(_i64p),
+                                int(nthreads))
+    if rc != 0:
+        raise IndexError(f"oracle prefill_attn: error {rc} (position or page id out of range)")
+    if full:
+        out = out.reshape(B, Tq, Hq, d)
     return (out, int(macs[0])) if return_macs else out

@@ -17,6 +17,10 @@
  *                    standard softmax attention.
  *   Sec. 3.2:        a dummy KV entry occupies cache slot 0, so the token at
  *                    position i is stored at slot i + 1.
+ *   Sec. 3.2-3.3:    causal attention for prefill and the token-parallel
+ *                    (Jacobi / cyclic Gauss-Seidel) passes: the query of the
+ *                    token at position i reads slots 0 .. i of its layer's
+ *                    channel, i.e. the dummy and the tokens before it.
  * Inputs are the same fp32 values, or bf16 bit patterns, the GPU receives;
  * they are widened to double on every read.
  *
@@ -302,6 +306,84 @@ int orc_decode_attn(int Hq, int Hkv, int d, int P, int num_pages, int max_pages,
     }
     for (int e = 0; e < d; ++e) o[e] /= wsum;
     m_attn += 2 * (int64_t)S * d;
+    free(s);
+    free(base);
+  }
+  if (macs) macs[0] += m_attn;
+  return err;
+}
+
+/*
+ * Sec. 3.1 Step 3 ("standard causal SDPA") with the dummy offset of Sec. 3.2,
+ * for many query positions at once: prefill, and one pass of the parallel
+ * schedules of Sec. 3.3 (Jacobi: every position; cyclic Gauss-Seidel: the
+ * strided group {i : i mod g = q}).  The dummy sits at slot 0 and token t at
+ * slot t + 1, so the query of the token at position i may read slots 0 .. i
+ * and never the channels at slot i + 1 that its own states produce.
+ *
+ * q is [B][Tq][Hq][d]: row r of sequence b is the query of the token at
+ * position pos[b][r].  For each listed unit (b, r, hq), with hkv = hq / (Hq/Hkv):
+ *   s_t = q . K[t] / sqrt(d) for t = 0 .. pos,  w_t = exp(s_t - max s),
+ *   o = sum_t w_t V[t] / sum_t w_t.
+ * Returns ORC_ERR_BOUNDS if a position is negative or beyond the page table,
+ * or a page id used is outside [0, num_pages).
+ */
+int orc_prefill_attn(int Hq, int Hkv, int d, int P, int num_pages, int max_pages, int chan,
+                     int dt, const void* k_pool, const void* v_pool, const int32_t* page_table,
+                     const int32_t* pos, int Tq, const void* q, int nunits, const int32_t* units,
+                     double* out, int64_t* macs, int nthreads) {
+  if (Hkv <= 0 || Hq % Hkv != 0 || Tq <= 0) return ORC_ERR_ARG;
+  int group = Hq / Hkv;
+  int err = ORC_OK;
+  int64_t m_attn = 0;
+#ifdef _OPENMP
+#pragma omp parallel for schedule(dynamic, 1) num_threads(nthreads > 0 ? nthreads : 1) \
+    reduction(+ : m_attn) reduction(max : err)
+#endif
+  for (int u = 0; u < nunits; ++u) {
+    int b = units[3 * u], r = units[3 * u + 1], hq = units[3 * u + 2];
+    int hkv = hq / group;
+    int i = pos[(int64_t)b * Tq + r];
+    double* o = out + (int64_t)u * d;
+    for (int e = 0; e < d; ++e) o[e] = 0.0;
+    int nslots = i + 1; /* slots 0 .. i */
+    if (i < 0 || (nslots + P - 1) / P > max_pages) {
+      err = ORC_ERR_BOUNDS;
+      continue;
+    }
+    double* s = (double*)malloc(sizeof(double) * nslots);
+    int64_t* base = (int64_t*)malloc(sizeof(int64_t) * nslots);
+    int bad = 0;
+    for (int t = 0; t < nslots; ++t) {
+      int32_t pg = page_table[(int64_t)b * max_pages + t / P];
+      if (pg < 0 || pg >= num_pages) {
+        bad = 1;
+        break;
+      }
+      base[t] = ((((int64_t)chan * num_pages + pg) * Hkv + hkv) * P + (t % P)) * d;
+    }
+    if (bad) {
+      err = ORC_ERR_BOUNDS;
+      free(s);
+      free(base);
+      continue;
+    }
+    int64_t qoff = (((int64_t)b * Tq + r) * Hq + hq) * d;
+    double scale = 1.0 / sqrt((double)d), smax = -INFINITY;
+    for (int t = 0; t < nslots; ++t) {
+      double acc = 0.0;
+      for (int e = 0; e < d; ++e) acc += rd(q, qoff + e, dt) * rd(k_pool, base[t] + e, dt);
+      s[t] = acc * scale;
+      if (s[t] > smax) smax = s[t];
+    }
+    double wsum = 0.0;
+    for (int t = 0; t < nslots; ++t) {
+      double wt = exp(s[t] - smax);
+      wsum += wt;
+      for (int e = 0; e < d; ++e) o[e] += wt * rd(v_pool, base[t] + e, dt);
+    }
+    for (int e = 0; e < d; ++e) o[e] /= wsum;
+    m_attn += 2 * (int64_t)nslots * d;
     free(s);
     free(base);
   }

@@ -157,6 +157,96 @@ def test_attention_rejects_bad_page_ids():
 
 # ---------------------------------------------------------------- RMSNorm/RoPE
 
+# ----------------------------------------------------- prefill attention (Sec. 3.2-3.3)
+
+def _prefill_case(rng, T, B, Hq, Hkv, d, P, permute):
+    """Channel caches holding the dummy and T tokens (slots 0..T) per sequence."""
+    kp, vp, pt = make_paged(rng, 2, [T + 1] * B, Hkv, d, P, permute)
+    return kp, vp, pt
+
+
+@pytest.mark.parametrize("Hq,Hkv,d,P,permute", [(4, 2, 8, 4, True), (2, 2, 16, 8, False),
+                                                (6, 3, 12, 16, True)])
+def test_prefill_matches_dense_masked_softmax(Hq, Hkv, d, P, permute):
+    """Sec. 3.2: causal SDPA over the dummy-offset cache, written as one dense
+    score matrix per head with the mask slot > position set to -inf."""
+    rng = np.random.default_rng(100 + d)
+    T, B = 37, 2
+    kp, vp, pt = _prefill_case(rng, T, B, Hq, Hkv, d, P, permute)
+    # rows at arbitrary positions (unsorted, repeated): any set of positions is one call
+    pos = np.stack([rng.permutation(T)[:20], rng.integers(0, T, 20)]).astype(np.int32)
+    q = rnd(rng, B, 20, Hq, d)
+    chan = 1
+    out = O.prefill_attn(q, kp, vp, pt, pos, chan=chan, Hq=Hq, Hkv=Hkv, d=d, P=P)
+    slots = np.arange(T + 1)
+    for b in range(B):
+        for hq in range(Hq):
+            hkv = hq // (Hq // Hkv)
+            K = gather(kp, chan, pt, b, hkv, T + 1, P)
+            V = gather(vp, chan, pt, b, hkv, T + 1, P)
+            S = q[b, :, hq].astype(np.float64) @ K.T / math.sqrt(d)      # [rows][slots]
+            S = np.where(slots[None, :] <= pos[b][:, None], S, -np.inf)
+            ref = scipy.special.softmax(S, axis=1) @ V
+            np.testing.assert_allclose(out[b, :, hq], ref, rtol=0, atol=1e-12)
+
+
+def test_prefill_position_zero_reads_only_the_dummy():
+    rng = np.random.default_rng(101)
+    kp, vp, pt = _prefill_case(rng, 9, 1, 2, 2, 8, 4, True)
+    q = rnd(rng, 1, 3, 2, 8, scale=5.0)
+    pos = np.zeros((1, 3), dtype=np.int32)
+    out = O.prefill_attn(q, kp, vp, pt, pos, chan=0, Hq=2, Hkv=2, d=8, P=4)
+    for r in range(3):
+        for h in range(2):
+            assert np.array_equal(out[0, r, h], vp[0, pt[0, 0], h, 0].astype(np.float64))
+
+
+def test_prefill_never_reads_the_queries_own_slot():
+    """Sec. 3.2: the token at position i must not read slot i + 1 (its own
+    channels).  A key planted there with a huge logit changes nothing; the
+    same key one slot earlier (slot i, the previous token) dominates."""
+    rng = np.random.default_rng(102)
+    T, P, d, i = 40, 8, 16, 23
+    kp, vp, pt = _prefill_case(rng, T, 1, 1, 1, d, P, True)
+    q = rnd(rng, 1, 1, 1, d)
+    qq = q[0, 0, 0].astype(np.float64)
+    big = (qq * 40.0 * math.sqrt(d) / qq.dot(qq)).astype(np.float32)
+    pos = np.array([[i]], dtype=np.int32)
+    base = O.prefill_attn(q, kp, vp, pt, pos, chan=0, Hq=1, Hkv=1, d=d, P=P)
+    own = kp.copy()
+    own[0, pt[0, (i + 1) // P], 0, (i + 1) % P] = big
+    assert np.array_equal(O.prefill_attn(q, own, vp, pt, pos, chan=0, Hq=1, Hkv=1, d=d, P=P), base)
+    prev = kp.copy()
+    prev[0, pt[0, i // P], 0, i % P] = big
+    got = O.prefill_attn(q, prev, vp, pt, pos, chan=0, Hq=1, Hkv=1, d=d, P=P)[0, 0, 0]
+    want = vp[0, pt[0, i // P], 0, i % P].astype(np.float64)
+    np.testing.assert_allclose(got, want, rtol=0, atol=1e-12 * (1 + np.abs(want).max()))
+
+
+def test_prefill_row_equals_decode_of_the_same_token():
+    """The token at position i decodes with i + 1 cache slots (Sec. 3.2): one
+    prefill row and one decode step of that token give the same output."""
+    rng = np.random.default_rng(103)
+    T, B, Hq, Hkv, d, P = 30, 3, 4, 2, 8, 4
+    kp, vp, pt = _prefill_case(rng, T, B, Hq, Hkv, d, P, True)
+    pos = np.array([[0, 5, 29], [17, 3, 11], [29, 28, 1]], dtype=np.int32)
+    q = rnd(rng, B, 3, Hq, d)
+    out = O.prefill_attn(q, kp, vp, pt, pos, chan=1, Hq=Hq, Hkv=Hkv, d=d, P=P)
+    for r in range(3):
+        dec = O.decode_attn(q[:, r], kp, vp, pt, pos[:, r] + 1, chan=1, Hq=Hq, Hkv=Hkv, d=d, P=P)
+        np.testing.assert_allclose(out[:, r], dec, rtol=0, atol=1e-13)
+
+
+def test_prefill_rejects_positions_beyond_the_table():
+    rng = np.random.default_rng(104)
+    kp, vp, pt = _prefill_case(rng, 7, 1, 1, 1, 8, 4, False)
+    q = rnd(rng, 1, 1, 1, 8)
+    with pytest.raises(IndexError):
+        O.prefill_attn(q, kp, vp, pt, np.array([[8]], np.int32), chan=0, Hq=1, Hkv=1, d=8, P=4)
+    with pytest.raises(IndexError):
+        O.prefill_attn(q, kp, vp, pt, np.array([[-1]], np.int32), chan=0, Hq=1, Hkv=1, d=8, P=4)
+
+
 def test_rmsnorm_unit_rms_scale_invariance_and_gain():
     rng = np.random.default_rng(7)
     x = rng.standard_normal(96) * 3.7

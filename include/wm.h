@@ -205,6 +205,34 @@ wm_status wm_decode_attn_flags(const wm_config* cfg, const wm_cache* cache, int3
                                int32_t* dev_status, void* stream);
 
 /*
+ * Causal channel attention of one layer for many query positions at once:
+ * prefill, and one pass of the token-parallel schedules (Sec. 3.1 Step 3
+ * "standard causal SDPA"; dummy offset of Sec. 3.2; Jacobi and cyclic
+ * Gauss-Seidel passes of Sec. 3.3, whose group q is the positions
+ * {i : i mod g = q}).  The dummy sits at slot 0 and token t at slot t + 1, so
+ * query row r of sequence b, the token at position i = pos[b*Tq + r],
+ * attends over slots 0..i of channel c(layer) (the dummy and the tokens
+ * before it, never its own slot i + 1), kv head hq / (Hq/Hkv):
+ *   out = softmax(q K^T / sqrt(d)) V, fp32 softmax and accumulation, bf16
+ *   probabilities into the P V product (tensor cores).
+ *   q          device bf16 [B][Tq][Hq][d], already normed and rotated
+ *   pos        device int32 [B][Tq], 0 <= pos < max_pages*page_size; any
+ *              order; slots 0..pos must hold that sequence's cache entries
+ *   page_table device int32 [B][max_pages]
+ *   out        device bf16 [B][Tq][Hq][d]
+ * No workspace.  Slots beyond the largest position of a 128-row tile may hold
+ * anything (NaN included).  bf16 caches only, page_size >= 8, B and Hq at
+ * most 65535 (else WM_ERR_UNSUPPORTED).  A bad position zero-fills that row
+ * and sets WM_ERR_BOUNDS; a bad page id reads zeros for its slots and sets
+ * WM_ERR_BOUNDS.  B = 0 or Tq = 0 is a no-op.  Launches chain with
+ * programmatic dependent launch like wm_decode_attn.
+ */
+wm_status wm_prefill_attn(const wm_config* cfg, const wm_cache* cache, int32_t layer,
+                          const void* q, const int32_t* pos, const int32_t* page_table,
+                          int32_t B, int32_t Tq, int32_t max_pages, void* out,
+                          int32_t* dev_status, void* stream);
+
+/*
  * Self-test of the kernels' failure detection (no counterpart in the paper).
  * Every pipeline wait in this library is bounded; when a wait runs out the
  * kernel writes WM_ERR_TIMEOUT to the status word and returns instead of

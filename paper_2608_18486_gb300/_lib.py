@@ -18,7 +18,7 @@ WM_DT_F32, WM_DT_BF16 = 0, 1
 
 EXPORTED = ["wm_status_string", "wm_config_check", "wm_cache_bytes", "wm_cache_alloc",
             "wm_kv_mix_workspace", "wm_kv_mix", "wm_decode_attn_workspace", "wm_decode_attn",
-            "wm_decode_attn_flags"]
+            "wm_decode_attn_flags", "wm_prefill_attn"]
 WM_ATTN_INPUTS_READY = 1
 
 
@@ -81,6 +81,9 @@ def lib():
         L.wm_decode_attn_flags.restype = ctypes.c_int
         L.wm_decode_attn_flags.argtypes = [cp, ctypes.POINTER(wm_cache), i32, vp, vp, vp, i32, i32,
                                            vp, vp, sz, ctypes.c_uint32, vp, vp]
+        L.wm_prefill_attn.restype = ctypes.c_int
+        L.wm_prefill_attn.argtypes = [cp, ctypes.POINTER(wm_cache), i32, vp, vp, vp, i32, i32, i32,
+                                      vp, vp, vp]
         _lib = L
     return _lib
 
@@ -166,6 +169,13 @@ def wm_decode_attn_flags(cfg, cache, layer, q, page_table, seq_lens, B, max_page
                                       _p(page_table), _p(seq_lens), int(B), int(max_pages),
                                       _p(out), _p(workspace), int(ws_bytes), int(flags),
                                       _p(dev_status), stream)
+
+
+def wm_prefill_attn(cfg, cache, layer, q, pos, page_table, B, Tq, max_pages, out, dev_status,
+                    stream) -> int:
+    return lib().wm_prefill_attn(ctypes.byref(cfg), ctypes.byref(cache), int(layer), _p(q), _p(pos),
+                                 _p(page_table), int(B), int(Tq), int(max_pages), _p(out),
+                                 _p(dev_status), stream)
 
 
 def wm_decode_attn_noalloc(cfg, cache, layer, q, page_table, seq_lens, B, max_pages, out,

@@ -43,6 +43,28 @@ size_t attn_smem_bytes(int stage_bytes, int dtype, int d, int G, int B);
 cudaError_t launch_decode_attn(const AttnParams& p, int stage_bytes, int dtype, int d, int G,
                                int grid, cudaStream_t s);
 
+// ------------------------------------------------------------ prefill attention
+struct PrefillLaunch {
+  const void* q;              // [B][Tq][Hq][d] bf16
+  const int32_t* pos;         // [B][Tq] token position of each query row
+  const int32_t* page_table;  // [B][max_pages]
+  void* out;                  // [B][Tq][Hq][d] bf16
+  int32_t* status;
+  const void* k_pool;         // whole pools, all channels: [k][num_pages][Hkv][P][d]
+  const void* v_pool;
+  int32_t B, Tq, Hq, Hkv, d, k, chan, num_pages, max_pages, P;
+};
+cudaError_t launch_prefill_attn(const PrefillLaunch& L, cudaStream_t s);
+
+// ------------------------------------------------------------ TMA tensor maps
+// 2-D map of a row-major bf16 matrix [rows][cols] with a row pitch of
+// pitch_elems elements (a multiple of 8), a box of 64 columns x box_rows
+// rows and 128-byte swizzle; elements outside the matrix read as zero.
+// `tm` points at a CUtensorMap.  False if the encoder is missing or refuses.
+bool tma_available();
+bool tma_map_bf16_2d(void* tm, const void* ptr, uint64_t rows, uint64_t cols, uint64_t pitch_elems,
+                     uint32_t box_rows);
+
 // ------------------------------------------------------------ KV pool (mix)
 constexpr int kMaxRopeHalf = 64;  // d/2 for d <= 128
 

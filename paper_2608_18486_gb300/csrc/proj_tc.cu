@@ -251,30 +251,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   }
 }
 
-PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
-  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-  if (!fn) {
-    void* ptr = nullptr;
-    cudaDriverEntryPointQueryResult q;
-    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault,
-                                         &q) == cudaSuccess &&
-        q == cudaDriverEntryPointSuccess)
-      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
-  }
-  return fn;
-}
-
 // Row-major bf16 matrix [rows][cols] as a 2-D tensor map with a 64 x box_rows box.
 bool encode_kmajor(CUtensorMap* tm, const void* ptr, uint64_t rows, uint64_t cols, uint32_t box_rows) {
-  auto fn = encode_fn();
-  if (!fn) return false;
-  cuuint64_t dims[2] = {cols, rows};
-  cuuint64_t strides[1] = {cols * 2};
-  cuuint32_t box[2] = {(cuuint32_t)kTcBK, box_rows};
-  cuuint32_t estr[2] = {1, 1};
-  return fn(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box,
-            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+  return tma_map_bf16_2d(tm, ptr, rows, cols, cols, box_rows);
 }
 
 uint32_t pow2_at_least(uint32_t x, uint32_t lo) {
@@ -338,7 +317,7 @@ int token_tile(int B) {  // tokens per MMA N tile: a multiple of 16, at most 256
 }
 
 bool proj_tc_supported(const MixParams& mp) {
-  return (mp.d == 64 || mp.d == 96 || mp.d == 128) && mp.B >= 1 && encode_fn() != nullptr;
+  return (mp.d == 64 || mp.d == 96 || mp.d == 128) && mp.B >= 1 && tma_available();
 }
 
 bool router_tc_supported(int B) { return B >= 1; }

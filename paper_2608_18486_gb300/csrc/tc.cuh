@@ -92,6 +92,25 @@ __device__ __forceinline__ uint64_t sdesc_kmajor_sw128(uint32_t smem_addr) {
   return d;
 }
 
+// Shared-memory matrix descriptor of an MN-major tile with 128-byte swizzle
+// (a B operand whose N index is contiguous, e.g. V stored [slot][d]): each
+// 128-byte row holds 64 consecutive N elements of one K index, 8 K rows form
+// a 1024-byte swizzle atom.  lbo = bytes between 64-element N blocks, sbo =
+// bytes between 8-row K groups.
+__device__ __forceinline__ uint64_t sdesc_mnmajor_sw128(uint32_t smem_addr, uint32_t lbo,
+                                                        uint32_t sbo) {
+  uint64_t d = 0;
+  d |= (uint64_t)((smem_addr >> 4) & 0x3FFFu);
+  d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;
+  d |= (uint64_t)((sbo >> 4) & 0x3FFFu) << 32;
+  d |= (uint64_t)1u << 46;
+  d |= (uint64_t)2u << 61;
+  return d;
+}
+
+// Instruction-descriptor bit: the B operand is MN-major (N contiguous).
+constexpr uint32_t kIdescBMajorMN = 1u << 16;
+
 // Instruction descriptor of kind::f16: fp32 accumulator, bf16 A and B, both
 // K-major, M x N tile.
 __host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N) {

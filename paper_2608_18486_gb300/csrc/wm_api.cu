@@ -222,6 +222,47 @@ wm_status wm_decode_attn_flags(const wm_config* c, const wm_cache* cache, int32_
   return e == cudaSuccess ? WM_OK : WM_ERR_CUDA;
 }
 
+wm_status wm_prefill_attn(const wm_config* c, const wm_cache* cache, int32_t layer,
+                          const void* q, const int32_t* pos, const int32_t* page_table,
+                          int32_t B, int32_t Tq, int32_t max_pages, void* out,
+                          int32_t* dev_status, void* stream) {
+  wm_status st = wm_config_check(c);
+  if (st != WM_OK) return st;
+  if ((st = check_cache(*c, cache)) != WM_OK) return st;
+  if (layer < 0 || layer >= c->L || B < 0 || Tq < 0 || max_pages < 1) return WM_ERR_INVALID_ARG;
+  if (c->dtype != WM_DT_BF16 || c->page_size < 8) return WM_ERR_UNSUPPORTED;
+  if (B > 65535 || c->Hq > 65535) return WM_ERR_UNSUPPORTED;
+  if ((int64_t)max_pages * c->page_size > INT32_MAX / 2) return WM_ERR_INVALID_ARG;
+  if ((int64_t)B * Tq >= INT32_MAX) return WM_ERR_UNSUPPORTED;
+  if ((int64_t)c->k * cache->num_pages * c->Hkv * c->page_size >= INT32_MAX)
+    return WM_ERR_UNSUPPORTED;  // TMA row coordinates are 32-bit
+  if (B == 0 || Tq == 0) return WM_OK;
+  if (!q || !pos || !page_table || !out) return WM_ERR_INVALID_ARG;
+  if (!aligned(q, 16) || !aligned(out, 16)) return WM_ERR_INVALID_ARG;
+  if (!wm::tma_available()) return WM_ERR_CUDA;
+  wm::PrefillLaunch L{};
+  L.q = q;
+  L.pos = pos;
+  L.page_table = page_table;
+  L.out = out;
+  L.status = dev_status;
+  L.k_pool = cache->k_pool;
+  L.v_pool = cache->v_pool;
+  L.B = B;
+  L.Tq = Tq;
+  L.Hq = c->Hq;
+  L.Hkv = c->Hkv;
+  L.d = c->d;
+  L.k = c->k;
+  L.chan = c->chan_of_layer[layer];
+  L.num_pages = cache->num_pages;
+  L.max_pages = max_pages;
+  L.P = c->page_size;
+  const cudaError_t e = wm::launch_prefill_attn(L, (cudaStream_t)stream);
+  if (e == cudaErrorInvalidValue) return WM_ERR_INVALID_ARG;  // the tensor-map encoder refused
+  return e == cudaSuccess ? WM_OK : WM_ERR_CUDA;
+}
+
 size_t wm_kv_mix_workspace(const wm_config* c, int32_t B) {
   if (wm_config_check(c) != WM_OK || B < 0) return 0;
   if (B == 0) return 256;

@@ -73,6 +73,15 @@ class DecodeSession:
         if rc != W.WM_OK:
             raise W.WMError(rc, "wm_decode_attn_flags")
 
+    def prefill_attn(self, layer: int, q, pos, page_table, out, stream=None) -> None:
+        """Causal attention of query rows q [B][Tq][Hq][d] at token positions
+        pos [B][Tq] over layer ``layer``'s channel (prefill / parallel passes)."""
+        B, Tq = int(q.shape[0]), int(q.shape[1])
+        rc = W.wm_prefill_attn(self.cfg, self.cache, layer, q, pos, page_table, B, Tq,
+                               self.max_pages, out, self.status, self._stream(stream))
+        if rc != W.WM_OK:
+            raise W.WMError(rc, "wm_prefill_attn")
+
     def kv_mix(self, h, page_table, slot, B: int | None = None, stream=None) -> None:
         if self._weights is None:
             raise RuntimeError("set_weights() first")

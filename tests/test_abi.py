@@ -99,3 +99,29 @@ def test_compute_calls_reject_bad_arguments_before_launching():
 def test_status_strings():
     for code in range(6):
         assert W.wm_status_string(code) and W.wm_status_string(code) != "unknown status"
+
+
+def test_prefill_rejects_unsupported_and_bad_arguments_before_launching():
+    c = cfg()
+    n = W.wm_cache_bytes(c, 4)
+    cache = W.wm_cache_alloc(c, 1 << 40, n, 4)
+    fake = 1 << 41
+    # fp32 caches and pages under 8 slots are not built
+    c32 = cfg(dtype=W.WM_DT_F32)
+    cache32 = W.wm_cache_alloc(c32, 1 << 40, W.wm_cache_bytes(c32, 4), 4)
+    assert W.wm_prefill_attn(c32, cache32, 0, fake, fake, fake, 2, 8, 4, fake, None,
+                             None) == W.WM_ERR_UNSUPPORTED
+    c4 = cfg(page_size=4)
+    cache4 = W.wm_cache_alloc(c4, 1 << 40, W.wm_cache_bytes(c4, 4), 4)
+    assert W.wm_prefill_attn(c4, cache4, 0, fake, fake, fake, 2, 8, 4, fake, None,
+                             None) == W.WM_ERR_UNSUPPORTED
+    # layer out of range, NULL positions, misaligned output
+    assert W.wm_prefill_attn(c, cache, c.L, fake, fake, fake, 2, 8, 4, fake, None,
+                             None) == W.WM_ERR_INVALID_ARG
+    assert W.wm_prefill_attn(c, cache, 0, fake, None, fake, 2, 8, 4, fake, None,
+                             None) == W.WM_ERR_INVALID_ARG
+    assert W.wm_prefill_attn(c, cache, 0, fake, fake, fake, 2, 8, 4, fake + 2, None,
+                             None) == W.WM_ERR_INVALID_ARG
+    # nothing to do is a no-op even with NULL buffers
+    assert W.wm_prefill_attn(c, cache, 0, None, None, None, 0, 8, 4, None, None, None) == W.WM_OK
+    assert W.wm_prefill_attn(c, cache, 0, None, None, None, 2, 0, 4, None, None, None) == W.WM_OK

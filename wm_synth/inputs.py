@@ -28,6 +28,7 @@ STREAM_WKV = 20
 STREAM_KPOOL = 30
 STREAM_VPOOL = 31
 STREAM_Q = 40
+STREAM_Q_PREFILL = 41
 
 
 @dataclass(frozen=True)
@@ -150,3 +151,16 @@ def make_problem(w: Workload, seed: int = 0, seq_lens=None) -> Problem:
         "q": TensorSpec(STREAM_Q, (w.L, w.B, w.Hq, w.d), w.q_scale),
     }
     return prob
+
+
+def prefill_queries(w: Workload, seed: int, B: int, Tq: int) -> np.ndarray:
+    """Query rows [B][Tq][Hq][d] of one prefill pass, stored in ``w.dtype``
+    (same distribution as the decode queries)."""
+    n = B * Tq * w.Hq * w.d
+    return gen.values(w.dtype, seed, STREAM_Q_PREFILL, 0, n, w.q_scale).reshape(B, Tq, w.Hq, w.d)
+
+
+def group_positions(T: int, g: int, q: int) -> np.ndarray:
+    """Token positions of strided group q of g over a T-token prefill:
+    {i : 0 <= i < T, i mod g = q} in increasing order (g = 1: all of them)."""
+    return np.arange(q, T, g, dtype=np.int32)

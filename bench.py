@@ -529,6 +529,99 @@ def run_model(args, w):
     print(json.dumps(line), flush=True)
 
 
+def gpu_uuid_of(dev, fallback):
+    import torch
+    u = str(getattr(torch.cuda.get_device_properties(dev), "uuid", "") or fallback)
+    if u and not u.startswith("GPU-") and len(u) > 8:
+        u = "GPU-" + u
+    return u
+
+
+def run_prefill(args, w):
+    """One prefill pass of causal channel attention over every layer (Sec. 3.2
+    dummy offset; Sec. 3.3 passes): for each layer, each of the g strided
+    Gauss-Seidel groups {i mod g = q} of the T-token prompt (g = 1: one Jacobi
+    pass) attends over its layer's channel.  The cache holds the dummy and T
+    tokens per sequence.  Prints one JSON line: prompt tokens/s of the pass and
+    the kernel's useful TFLOP/s (causal FLOPs only) against the measured bf16
+    tensor peak."""
+    import numpy as np
+    import torch
+    from paper_2608_18486_gb300 import make_config
+    from paper_2608_18486_gb300.session import DecodeSession
+    from wm_synth import device as wdev
+    from wm_synth.device_problem import DeviceProblem
+    from wm_synth.inputs import STREAM_Q_PREFILL, group_positions, make_problem
+
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    T, g = w.ctx, args.groups
+    prob = make_problem(w, seed=0, seq_lens=[T] * w.B)
+    cfg = make_config(w.L, w.k, w.D, w.Hq, w.Hkv, w.d, w.p, w.page, w.dtype, w.chan_of_layer(),
+                      w.eps_rms, w.eps_qk, w.rope_theta)
+    sess = DecodeSession(cfg, w.B, prob.num_pages, prob.max_pages, dev)
+    dp = DeviceProblem(prob, sess.k_pool, sess.v_pool, dev)
+    groups = []
+    start_idx = 0
+    for q in range(g):
+        pos = torch.from_numpy(np.stack([group_positions(T, g, q)] * w.B)).to(dev)
+        Tq = pos.shape[1]
+        qt = torch.empty((w.B, Tq, w.Hq, w.d), dtype=sess.dtype, device=dev)
+        wdev.fill(qt, w.dtype, 0, STREAM_Q_PREFILL, w.q_scale, 0.0, start=start_idx)
+        start_idx += qt.numel()
+        groups.append((qt, pos, torch.empty_like(qt)))
+    stream = torch.cuda.Stream(dev)
+
+    def step():
+        for layer in range(w.L):
+            for qt, pos, out in groups:
+                sess.prefill_attn(layer, qt, pos, dp.page_table, out, stream=stream)
+
+    with torch.cuda.stream(stream):
+        for _ in range(args.warmup):
+            step()
+    torch.cuda.synchronize()
+    if sess.read_status() != 0:
+        raise RuntimeError("device status set during warm-up")
+    K = args.steps
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=stream):
+        for _ in range(K):
+            step()
+    with torch.cuda.stream(stream):
+        graph.replay()
+    torch.cuda.synchronize()
+    sampler = ClockSampler(gpu_uuid_of(dev, "0"))
+    time.sleep(0.3)
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t0 = time.time()
+    with torch.cuda.stream(stream):
+        start.record(stream)
+        graph.replay()
+        end.record(stream)
+    torch.cuda.synchronize()
+    t1 = time.time()
+    clocks = sampler.stop(t0, t1)
+    if sess.read_status() != 0:
+        raise RuntimeError("device status set during the timed region")
+    ms = start.elapsed_time(end) / K
+    flops = w.L * w.B * w.Hq * 4.0 * w.d * (T * (T + 1) / 2.0)  # sum over positions of pos + 1
+    tflops = flops / (ms * 1e-3) / 1e12
+    peaks = json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
+    peak = float(peaks["bf16_tflops_sustained"])
+    line = {"metric": "prefill attention tokens/s (one pass over all layers; causal channel attention)",
+            "value": w.B * T / (ms * 1e-3), "unit": "tokens/s", "n_gpus": 1, "steps": K,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "dtype": "bf16",
+            "data": "synthetic",
+            "config": dict(config_dict(w, 1), mode="prefill", prompt_tokens=T, groups=g,
+                           launches_per_step=w.L * g),
+            "roofline": {"bound": "tensor", "achieved": tflops, "peak": peak, "unit": "TFLOP/s",
+                         "frac": tflops / peak, "peak_kind": "measured sustained bf16",
+                         "flops_per_step": flops},
+            "clocks": clocks, "gpu_launches": K * w.L * g}
+    print(json.dumps(line), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -536,8 +629,11 @@ def main():
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
-    ap.add_argument("--mode", default="path", choices=["path", "model"],
-                    help="path: the WhiteMatter hot path (default); model: a whole-model step")
+    ap.add_argument("--mode", default="path", choices=["path", "model", "prefill"],
+                    help="path: the WhiteMatter decode hot path (default); model: a whole-model "
+                         "decode step; prefill: causal channel attention of a prefill pass")
+    ap.add_argument("--groups", type=int, default=8,
+                    help="--mode prefill: strided Gauss-Seidel groups (1: a Jacobi pass)")
     ap.add_argument("--intermediate", type=int, default=0,
                     help="MLP width for --mode model (default 3*D)")
     ap.add_argument("--ref-budget", type=float, default=4.0,
@@ -559,6 +655,8 @@ def main():
         run_reference(args, w)
     elif args.mode == "model":
         run_model(args, w)
+    elif args.mode == "prefill":
+        run_prefill(args, w)
     else:
         run_gpu(args, w)
 

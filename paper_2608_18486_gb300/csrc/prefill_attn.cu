@@ -6,22 +6,25 @@
 //
 // Design (GB300).  A prefill pass is a dense contraction on both sides of the
 // softmax, so it runs on the tcgen05 tensor cores (bf16 operands, fp32
-// accumulation in TMEM).  One CTA (4 warps) owns 128 query rows of one query
-// head and walks the 128-slot KV tiles of the sequence's channel up to the
-// tile's largest position:
-//  * TMA brings the Q tile once and the K and V tiles of each KV tile
-//    (128-byte swizzle, 64-column boxes; paged: one box per page or per 128
-//    slots of a page) through a 2-deep stage ring;
-//  * S = Q K^T lands in TMEM columns [0, 128); each thread owns one query row
-//    (its TMEM lane), applies the causal mask slot <= pos, keeps the running
-//    max and sum, and writes the bf16 probabilities P into shared memory in
-//    the layout of an MMA A operand;
-//  * O_tile = P V lands in TMEM columns [128, 128 + d) (V is read as an
-//    MN-major B operand straight from its [slot][d] tile); each thread folds
-//    its row into registers with the softmax correction;
-//  * S of the next KV tile is issued right behind P V, so the tensor core
-//    works on it while the threads drain O_tile.
-// Slots beyond the tile's largest position may hold anything (unwritten
+// accumulation in TMEM), warp-specialised in the manner of flash attention on
+// this architecture.  One CTA (10 warps, one per SM) owns two 128-row query
+// tiles of one query head and walks the 128-slot KV tiles of the sequence's
+// channel up to each tile's largest position:
+//  * warp 8 (TMA): the two Q tiles once, then K and V of every KV tile
+//    through separate rings (128-byte swizzle, 64-column boxes; paged: one
+//    box per page, or per 128 slots of a longer page);
+//  * warp 9 (MMA): S_i = Q_i K^T into TMEM, and O_i += P_i V with P_i read
+//    from TMEM and V as an MN-major operand straight from its [slot][d] tile;
+//    issue order PV_0(j), S_0(j+1), PV_1(j), S_1(j+1) keeps one tile's
+//    matrix products running while the other tile's softmax works;
+//  * warps 0-3 and 4-7 (softmax of tile 0 / 1): one thread per query row
+//    reads its S row from TMEM, applies the causal mask slot <= pos (on
+//    tiles the diagonal crosses), and writes the bf16 probabilities back over
+//    the S columns it has read, where P V takes them as its A operand.  The
+//    running max is raised only when it grows by more than 2^8: only then is
+//    the row of O in TMEM rescaled; in between the probabilities stay below
+//    2^8, and the final O / l is exact either way.
+// Slots beyond the CTA's largest position may hold anything (unwritten
 // cache); their V rows are zeroed in shared memory before P V, and masked
 // scores are replaced, never multiplied, so no NaN there reaches the output.
 #include <math.h>
@@ -32,21 +35,25 @@
 namespace wm {
 namespace {
 
-constexpr int kPM = 128;         // query rows per CTA (MMA M)
-constexpr int kPN = 128;         // slots per KV tile
-constexpr int kPThreads = 128;   // one thread per query row
-constexpr uint32_t kBlock = 128u * 128u;  // one 64-column block of a 128-row tile
+constexpr int kPM = 128;                    // query rows per tile (MMA M)
+constexpr int kPN = 128;                    // slots per KV tile
+constexpr int kQT = 2;                      // query tiles per CTA
+constexpr int kSoftWarps = 4 * kQT;         // one 4-warp group per query tile
+constexpr int kLoadWarp = kSoftWarps;       // TMA producer
+constexpr int kMmaWarp = kSoftWarps + 1;    // MMA issuer
+constexpr int kPThreads = (kSoftWarps + 2) * 32;
+constexpr uint32_t kBlock = 128u * 128u;    // one 64-column block of a 128-row tile
+constexpr uint32_t kTmemCols = 512;         // S_i at 128 i (P_i over its first 64), O_i at 256 + 128 i
+constexpr float kStaleMax = 8.f;            // log2 headroom before O is rescaled
 
 template <int HD>
 struct PShape {
-  static constexpr int CB = (HD + 63) / 64;                   // 64-column blocks of a head row
-  static constexpr uint32_t Q_BYTES = CB * kBlock;
-  static constexpr uint32_t KV_BYTES = CB * kBlock;           // one K or V tile
-  static constexpr uint32_t STAGE = 2 * KV_BYTES;             // K then V
-  static constexpr uint32_t P_BYTES = 2 * kBlock;             // 128 x 128 bf16
-  static constexpr uint32_t SMEM = Q_BYTES + 2 * STAGE + P_BYTES + 1024;  // + alignment
+  static constexpr int CB = (HD + 63) / 64;          // 64-column blocks of a head row
+  static constexpr int NST = HD <= 64 ? 3 : 2;       // depth of the K and V rings
+  static constexpr uint32_t Q_BYTES = CB * kBlock;   // one Q tile
+  static constexpr uint32_t KV_BYTES = CB * kBlock;  // one K or V tile
+  static constexpr uint32_t SMEM = kQT * Q_BYTES + 2 * NST * KV_BYTES + 1024;  // + alignment
 };
-constexpr uint32_t kPTmemCols = 256;  // S in [0, 128), O_tile in [128, 128 + d)
 
 struct PrefillParams {
   const int32_t* pos;         // [B][Tq]
@@ -57,14 +64,10 @@ struct PrefillParams {
   float qscale;               // log2(e) / sqrt(d)
 };
 
-__device__ __forceinline__ int block_max(int v, int* red) {
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v = max(v, __shfl_xor_sync(0xFFFFFFFFu, v, o));
-  __syncthreads();
-  if (lane == 0) red[warp] = v;
-  __syncthreads();
-  return max(max(red[0], red[1]), max(red[2], red[3]));
+__device__ __forceinline__ float ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
 }
 
 template <int HD>
@@ -73,36 +76,43 @@ __global__ void __launch_bounds__(kPThreads, 1)
                         const __grid_constant__ CUtensorMap tmK,
                         const __grid_constant__ CUtensorMap tmV, const PrefillParams p) {
   using SH = PShape<HD>;
-  constexpr int CB = SH::CB;
+  constexpr int CB = SH::CB, NST = SH::NST;
   extern __shared__ uint8_t smem_dyn[];
-  __shared__ uint64_t qbar, full[2], sbar, obar;
+  __shared__ uint64_t qbar, kfull[NST], kempty[NST], vfull[NST], vempty[NST];
+  __shared__ uint64_t sfull[kQT], pfull[kQT], odone[kQT];
   __shared__ uint32_t tmem_base;
-  __shared__ int red[4];
+  __shared__ int wmax[kSoftWarps];
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int b = blockIdx.z, hq = blockIdx.y, hkv = hq / p.G;
-  const int ntiles = (p.Tq + kPM - 1) / kPM;
-  const int r0 = (ntiles - 1 - (int)blockIdx.x) * kPM;  // later rows (more work) start first
-  const int r = r0 + tid;
+  const int nblk = (p.Tq + kQT * kPM - 1) / (kQT * kPM);
+  const int r0 = (nblk - 1 - (int)blockIdx.x) * kQT * kPM;  // later rows (more work) first
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_dyn) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
-  uint8_t* Qs = base;
-  uint8_t* KVs = Qs + SH::Q_BYTES;  // [2 stages][K | V]
-  uint8_t* Ps = KVs + 2 * SH::STAGE;
+  uint8_t* Qs = base;                         // [kQT] Q tiles
+  uint8_t* Ks = Qs + kQT * SH::Q_BYTES;       // [NST] K tiles
+  uint8_t* Vs = Ks + NST * SH::KV_BYTES;      // [NST] V tiles
 
   if (tid == 0) {
     mbar_init(&qbar, 1);
-    mbar_init(&full[0], 1);
-    mbar_init(&full[1], 1);
-    mbar_init(&sbar, 1);
-    mbar_init(&obar, 1);
+    for (int s = 0; s < NST; ++s) {
+      mbar_init(&kfull[s], 1);
+      mbar_init(&kempty[s], 1);
+      mbar_init(&vfull[s], 1);
+      mbar_init(&vempty[s], 1);
+    }
+    for (int i = 0; i < kQT; ++i) {
+      mbar_init(&sfull[i], 1);
+      mbar_init(&pfull[i], kPM);
+      mbar_init(&odone[i], 1);
+    }
     fence_mbar_init();
     tc::prefetch_tensormap(&tmQ);
     tc::prefetch_tensormap(&tmK);
     tc::prefetch_tensormap(&tmV);
   }
   if (warp == 0) {
-    tc::tmem_alloc(&tmem_base, kPTmemCols);
+    tc::tmem_alloc(&tmem_base, kTmemCols);
     tc::tmem_relinquish();
   }
   // programmatic dependent launch: positions, table, queries and cache may
@@ -110,195 +120,277 @@ __global__ void __launch_bounds__(kPThreads, 1)
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   asm volatile("griddepcontrol.wait;" ::: "memory");
 
+  // ---- positions of the softmax threads' rows; the largest of each tile
   const int max_slots = p.max_pages * p.P;
   int mypos = -1;  // -1: row absent or invalid, fully masked
-  if (r < p.Tq) {
+  const int r = r0 + tid;
+  if (warp < kSoftWarps && r < p.Tq) {
     const int v = p.pos[(int64_t)b * p.Tq + r];
     if (v >= 0 && v < max_slots) mypos = v;
     else report(p.status, WM_ERR_BOUNDS);
   }
+  if (warp < kSoftWarps) {
+    int mx = mypos;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      mx = max(mx, __shfl_xor_sync(0xFFFFFFFFu, mx, o));
+    }
+    if (lane == 0) {
+      wmax[warp] = mx;
+    }
+  }
   tc::fence_before_sync();
-  const int maxpos = block_max(mypos, red);  // also publishes the barrier inits and TMEM base
+  __syncthreads();
   tc::fence_after_sync();
   const uint32_t tmem = tmem_base;
-  const int nkv = maxpos >= 0 ? maxpos / kPN + 1 : 0;  // KV tiles 0 .. nkv-1
-
-  // ---- producer (thread 0): K and V of KV tile j into stage j & 1
-  auto issue_kv = [&](int j) {
-    const int st = j & 1;
-    uint8_t* Kd = KVs + st * SH::STAGE;
-    uint8_t* Vd = Kd + SH::KV_BYTES;
-    mbar_arrive_expect_tx(&full[st], SH::STAGE);
-    const int s0 = j * kPN;
-    const int boxes = p.P >= kPN ? 1 : kPN >> p.log2P;
-    const int brows = p.P >= kPN ? kPN : p.P;
-    for (int t = 0; t < boxes; ++t) {
-      const int s = s0 + t * brows;        // first slot of the box
-      const int lp = s >> p.log2P;         // logical page
-      int row = -brows;                    // fully outside the map: reads zeros
-      if (s <= maxpos && lp < p.max_pages) {
-        const int pg = p.page_table[(int64_t)b * p.max_pages + lp];
-        if (pg >= 0 && pg < p.num_pages)
-          row = (int)((((int64_t)p.chan * p.num_pages + pg) * p.Hkv + hkv) * p.P + (s & (p.P - 1)));
-        else
-          report(p.status, WM_ERR_BOUNDS);
-      }
+  int ntile[kQT], tmaxpos = -1;
 #pragma unroll
-      for (int cb = 0; cb < CB; ++cb) {
-        tc::tma_load_2d(Kd + cb * kBlock + t * brows * 128, &tmK, cb * 64, row, &full[st]);
-        tc::tma_load_2d(Vd + cb * kBlock + t * brows * 128, &tmV, cb * 64, row, &full[st]);
-      }
-    }
-  };
-  const uint32_t idesc_s = tc::idesc_bf16_f32(kPM, kPN);
-  const uint32_t idesc_o = tc::idesc_bf16_f32(kPM, HD) | tc::kIdescBMajorMN;
-  auto issue_s = [&](int j) {  // S = Q K_j^T into TMEM columns [0, 128)
-    const uint32_t q0 = smem_u32(Qs), k0 = smem_u32(KVs + (j & 1) * SH::STAGE);
-#pragma unroll
-    for (int kk = 0; kk < HD / 16; ++kk) {
-      const uint32_t off = (kk >> 2) * kBlock + (kk & 3) * 32;
-      tc::mma_bf16(tmem, tc::sdesc_kmajor_sw128(q0 + off), tc::sdesc_kmajor_sw128(k0 + off),
-                   idesc_s, kk > 0);
-    }
-    tc::mma_commit(&sbar);
-  };
-  auto issue_o = [&](int j) {  // O_tile = P V_j into TMEM columns [128, 128 + HD)
-    const uint32_t p0 = smem_u32(Ps), v0 = smem_u32(KVs + (j & 1) * SH::STAGE + SH::KV_BYTES);
-#pragma unroll
-    for (int kk = 0; kk < kPN / 16; ++kk) {
-      const uint64_t adesc = tc::sdesc_kmajor_sw128(p0 + (kk >> 2) * kBlock + (kk & 3) * 32);
-      const uint64_t bdesc = tc::sdesc_mnmajor_sw128(v0 + kk * 16 * 128, kBlock, 1024);
-      tc::mma_bf16(tmem + kPM, adesc, bdesc, idesc_o, kk > 0);
-    }
-    tc::mma_commit(&obar);
-  };
-
-  bool ok = true;
-  if (tid == 0 && nkv > 0) {
-    mbar_arrive_expect_tx(&qbar, SH::Q_BYTES);
-#pragma unroll
-    for (int cb = 0; cb < CB; ++cb)
-      tc::tma_load_2d(Qs + cb * kBlock, &tmQ, hq * HD + cb * 64, b * p.Tq + r0, &qbar);
-    issue_kv(0);
-    if (nkv > 1) issue_kv(1);
-    ok = mbar_wait(&qbar, 0) && mbar_wait(&full[0], 0);
-    if (ok) {
-      tc::fence_after_sync();
-      issue_s(0);
-    }
+  for (int i = 0; i < kQT; ++i) {
+    const int mx = max(max(wmax[4 * i], wmax[4 * i + 1]), max(wmax[4 * i + 2], wmax[4 * i + 3]));
+    ntile[i] = mx >= 0 ? mx / kPN + 1 : 0;  // KV tiles of query tile i
+    tmaxpos = max(tmaxpos, mx);
   }
+  const int nmax = tmaxpos >= 0 ? tmaxpos / kPN + 1 : 0;
 
-  float m = -INFINITY, l = 0.f;  // running max (log2 units) and sum of this row
-  float o[HD];
-#pragma unroll
-  for (int i = 0; i < HD; ++i) o[i] = 0.f;
-  const uint32_t lane_base = tmem + ((uint32_t)(warp * 32) << 16);
-  uint8_t* prow = Ps + tid * 128;
-  const int sw = tid & 7;  // 128-byte swizzle: 16-byte unit u of row t sits at u ^ (t & 7)
-
-  for (int j = 0; j < nkv; ++j) {
-    ok = __syncthreads_and(ok);
-    if (!ok) break;
-    ok = mbar_wait(&sbar, j & 1);
-    tc::fence_after_sync();
-    const int s0 = j * kPN;
-    // pass 1: row max of the masked, scaled scores
-    float mx = -INFINITY;
-#pragma unroll
-    for (int c = 0; c < kPN / 16; ++c) {
-      uint32_t v[16];
-      tc::tmem_ld16(lane_base + c * 16, v);
-      tc::tmem_ld_wait();
-#pragma unroll
-      for (int i = 0; i < 16; ++i)
-        if (s0 + c * 16 + i <= mypos) mx = fmaxf(mx, __uint_as_float(v[i]) * p.qscale);
-    }
-    const float mn = fmaxf(m, mx);
-    const float corr = (m == -INFINITY) ? 0.f : exp2f(m - mn);
-    // pass 2: probabilities (bf16) into the P tile, and their sum
-    float sum = 0.f;
-#pragma unroll
-    for (int c = 0; c < kPN / 16; ++c) {
-      uint32_t v[16];
-      tc::tmem_ld16(lane_base + c * 16, v);
-      tc::tmem_ld_wait();
-      uint32_t packed[8];
-#pragma unroll
-      for (int i = 0; i < 16; i += 2) {
-        const bool in0 = s0 + c * 16 + i <= mypos, in1 = s0 + c * 16 + i + 1 <= mypos;
-        const float p0 = in0 ? exp2f(__uint_as_float(v[i]) * p.qscale - mn) : 0.f;
-        const float p1 = in1 ? exp2f(__uint_as_float(v[i + 1]) * p.qscale - mn) : 0.f;
-        const __nv_bfloat162 h = __floats2bfloat162_rn(p0, p1);
-        sum += __low2float(h) + __high2float(h);
-        packed[i / 2] = *reinterpret_cast<const uint32_t*>(&h);
-      }
-      // columns 16c .. 16c+15: K block c/4, 16-byte units 2(c%4) and 2(c%4)+1
-      uint8_t* blk = prow + (c >> 2) * kBlock;
-      const int u = (c & 3) * 2;
-      *reinterpret_cast<uint4*>(blk + (((u) ^ sw) << 4)) =
-          make_uint4(packed[0], packed[1], packed[2], packed[3]);
-      *reinterpret_cast<uint4*>(blk + (((u + 1) ^ sw) << 4)) =
-          make_uint4(packed[4], packed[5], packed[6], packed[7]);
-    }
-    l = l * corr + sum;
-    m = mn;
-    if (j == nkv - 1 && s0 + kPN - 1 > maxpos) {
-      // slots past the largest position may be unwritten: zero their V rows
-      ok = mbar_wait(&full[j & 1], (j >> 1) & 1) && ok;
-      if (tid > maxpos - s0) {
-        uint8_t* vrow = KVs + (j & 1) * SH::STAGE + SH::KV_BYTES + tid * 128;
+  if (warp == kLoadWarp) {
+    // ================================================================ TMA
+    if (lane == 0 && nmax > 0) {
+      bool ok = true;
+      mbar_arrive_expect_tx(&qbar, kQT * SH::Q_BYTES);
+      for (int i = 0; i < kQT; ++i)
 #pragma unroll
         for (int cb = 0; cb < CB; ++cb)
+          tc::tma_load_2d(Qs + i * SH::Q_BYTES + cb * kBlock, &tmQ, hq * HD + cb * 64,
+                          b * p.Tq + r0 + i * kPM, &qbar);
+      const int boxes = p.P >= kPN ? 1 : kPN >> p.log2P;
+      const int brows = p.P >= kPN ? kPN : p.P;
+      auto load_tile = [&](const CUtensorMap* tm, uint8_t* dst, int j, uint64_t* bar) {
+        mbar_arrive_expect_tx(bar, SH::KV_BYTES);
+        const int s0 = j * kPN;
+        for (int t = 0; t < boxes; ++t) {
+          const int s = s0 + t * brows;  // first slot of the box
+          const int lp = s >> p.log2P;   // logical page
+          int row = -brows;              // fully outside the map: reads zeros
+          if (s <= tmaxpos && lp < p.max_pages) {
+            const int pg = p.page_table[(int64_t)b * p.max_pages + lp];
+            if (pg >= 0 && pg < p.num_pages)
+              row = (int)((((int64_t)p.chan * p.num_pages + pg) * p.Hkv + hkv) * p.P +
+                          (s & (p.P - 1)));
+            else
+              report(p.status, WM_ERR_BOUNDS);
+          }
 #pragma unroll
-          for (int u = 0; u < 8; ++u)
-            *reinterpret_cast<uint4*>(vrow + cb * kBlock + u * 16) = make_uint4(0, 0, 0, 0);
+          for (int cb = 0; cb < CB; ++cb)
+            tc::tma_load_2d(dst + cb * kBlock + t * brows * 128, tm, cb * 64, row, bar);
+        }
+      };
+      for (int j = 0; j < nmax && ok; ++j) {
+        const int st = j % NST, use = j / NST;
+        if (j >= NST) ok = mbar_wait(&kempty[st], (use - 1) & 1);
+        if (!ok) break;
+        load_tile(&tmK, Ks + st * SH::KV_BYTES, j, &kfull[st]);
+        if (j >= NST) ok = mbar_wait(&vempty[st], (use - 1) & 1);
+        if (!ok) break;
+        load_tile(&tmV, Vs + st * SH::KV_BYTES, j, &vfull[st]);
       }
+      if (!ok) report(p.status, WM_ERR_TIMEOUT);
     }
-    fence_proxy_async_shared();  // P (and zeroed V rows) visible to the tensor core
-    tc::fence_before_sync();
-    ok = __syncthreads_and(ok);
-    if (!ok) break;
-    if (tid == 0) {
+  } else if (warp == kMmaWarp) {
+    // ================================================================ MMA
+    // every lane runs the schedule (all wait, all zero the last V tile's
+    // unwritten rows, wait outcomes made warp-uniform); lane 0 issues
+    const uint32_t idesc_s = tc::idesc_bf16_f32(kPM, kPN);
+    const uint32_t idesc_o = tc::idesc_bf16_f32(kPM, HD) | tc::kIdescBMajorMN;
+    auto wait_all = [&](uint64_t* bar, uint32_t parity) {
+      return __all_sync(0xFFFFFFFFu, mbar_wait(bar, parity));
+    };
+    bool ok = nmax == 0 || wait_all(&qbar, 0);
+    auto issue_s = [&](int i, int j) {  // S_i = Q_i K_j^T
+      if (lane == 0) {
+        const uint32_t q0 = smem_u32(Qs + i * SH::Q_BYTES);
+        const uint32_t k0 = smem_u32(Ks + (j % NST) * SH::KV_BYTES);
+#pragma unroll
+        for (int kk = 0; kk < HD / 16; ++kk) {
+          const uint32_t off = (kk >> 2) * kBlock + (kk & 3) * 32;
+          tc::mma_bf16(tmem + 128 * i, tc::sdesc_kmajor_sw128(q0 + off),
+                       tc::sdesc_kmajor_sw128(k0 + off), idesc_s, kk > 0);
+        }
+        tc::mma_commit(&sfull[i]);
+      }
+    };
+    auto issue_pv = [&](int i, int j) {  // O_i += P_i V_j
+      if (lane == 0) {
+        const uint32_t v0 = smem_u32(Vs + (j % NST) * SH::KV_BYTES);
+#pragma unroll
+        for (int kk = 0; kk < kPN / 16; ++kk)
+          tc::mma_bf16_ts(tmem + 256 + 128 * i, tmem + 128 * i + 8 * kk,
+                          tc::sdesc_mnmajor_sw128(v0 + kk * 16 * 128, kBlock, 1024), idesc_o,
+                          (j | kk) != 0);
+        tc::mma_commit(&odone[i]);
+      }
+    };
+    if (ok && nmax > 0) {
+      ok = wait_all(&kfull[0], 0);
       tc::fence_after_sync();
-      issue_o(j);
-      if (j + 1 < nkv) {
-        ok = mbar_wait(&full[(j + 1) & 1], ((j + 1) >> 1) & 1);
-        tc::fence_after_sync();
-        if (ok) issue_s(j + 1);
+      if (ok) {
+        for (int i = 0; i < kQT; ++i)
+          if (ntile[i] > 0) issue_s(i, 0);
+        if (lane == 0) tc::mma_commit(&kempty[0]);
       }
     }
-    ok = mbar_wait(&obar, j & 1) && ok;
-    tc::fence_after_sync();
+    for (int j = 0; j < nmax && ok; ++j) {
+      const int st = j % NST;
+      ok = wait_all(&vfull[st], (j / NST) & 1);
+      if (!ok) break;
+      const int s0 = j * kPN;
+      if (j == nmax - 1 && s0 + kPN - 1 > tmaxpos) {
+        // slots past the largest position may be unwritten: zero their V rows
+        uint8_t* vt = Vs + st * SH::KV_BYTES;
+        for (int row = tmaxpos - s0 + 1 + lane; row < kPN; row += 32)
 #pragma unroll
-    for (int c = 0; c < HD / 16; ++c) {
-      uint32_t v[16];
-      tc::tmem_ld16(lane_base + kPM + c * 16, v);
-      tc::tmem_ld_wait();
+          for (int cb = 0; cb < CB; ++cb)
 #pragma unroll
-      for (int i = 0; i < 16; ++i) o[c * 16 + i] = fmaf(o[c * 16 + i], corr, __uint_as_float(v[i]));
+            for (int u = 0; u < 8; ++u)
+              *reinterpret_cast<uint4*>(vt + cb * kBlock + row * 128 + u * 16) =
+                  make_uint4(0, 0, 0, 0);
+        fence_proxy_async_shared();
+        __syncwarp();
+      }
+      const bool more = j + 1 < nmax;
+      if (more) {
+        ok = wait_all(&kfull[(j + 1) % NST], ((j + 1) / NST) & 1);
+        if (!ok) break;
+      }
+      for (int i = 0; i < kQT && ok; ++i) {
+        if (j >= ntile[i]) continue;
+        ok = wait_all(&pfull[i], j & 1);
+        if (!ok) break;
+        tc::fence_after_sync();
+        issue_pv(i, j);
+        if (j + 1 < ntile[i]) issue_s(i, j + 1);
+      }
+      if (lane == 0) {
+        tc::mma_commit(&vempty[st]);
+        if (more) tc::mma_commit(&kempty[(j + 1) % NST]);
+      }
+      __syncwarp();
     }
-    tc::fence_before_sync();
-    // stage j & 1 is free (S_j and P V_j are done): bring KV tile j + 2
-    if (tid == 0 && j + 2 < nkv && ok) issue_kv(j + 2);
-  }
-  if (!ok) {
-    report(p.status, WM_ERR_TIMEOUT);
-  } else if (r < p.Tq) {
-    const float inv = l > 0.f ? 1.f / l : 0.f;
-    __nv_bfloat16* dst =
-        reinterpret_cast<__nv_bfloat16*>(p.out) + (((int64_t)b * p.Tq + r) * p.Hq + hq) * HD;
+    if (!ok && lane == 0) report(p.status, WM_ERR_TIMEOUT);
+  } else {
+    // ================================================================ softmax
+    const int i = warp >> 2;  // query tile
+    const int n = ntile[i];
+    const uint32_t lane_base = tmem + ((uint32_t)((warp & 3) * 32) << 16);
+    const uint32_t scol = 128 * i, ocol = 256 + 128 * i;
+    float m = -INFINITY, l = 0.f;  // max used for P (log2 units) and running sum
+    bool ok = true;
+    // tcgen05.ld / st are warp-collective: every lane of the warp issues each
+    // one, and the wait outcomes are made warp-uniform before any branch
+    for (int j = 0; j < n && ok; ++j) {
+      ok = __all_sync(0xFFFFFFFFu, mbar_wait(&sfull[i], j & 1));
+      if (!ok) break;
+      tc::fence_after_sync();
+      const int s0 = j * kPN;
+      const bool full = s0 + kPN - 1 <= mypos;  // every slot of the tile is visible
+      float mx = -INFINITY;
 #pragma unroll
-    for (int i = 0; i < HD; i += 8) {
-      uint4 w;
-      __nv_bfloat162 t0 = __floats2bfloat162_rn(o[i] * inv, o[i + 1] * inv);
-      __nv_bfloat162 t1 = __floats2bfloat162_rn(o[i + 2] * inv, o[i + 3] * inv);
-      __nv_bfloat162 t2 = __floats2bfloat162_rn(o[i + 4] * inv, o[i + 5] * inv);
-      __nv_bfloat162 t3 = __floats2bfloat162_rn(o[i + 6] * inv, o[i + 7] * inv);
-      w.x = *reinterpret_cast<uint32_t*>(&t0);
-      w.y = *reinterpret_cast<uint32_t*>(&t1);
-      w.z = *reinterpret_cast<uint32_t*>(&t2);
-      w.w = *reinterpret_cast<uint32_t*>(&t3);
-      *reinterpret_cast<uint4*>(dst + i) = w;
+      for (int c = 0; c < kPN / 32; ++c) {
+        uint32_t v[32];
+        tc::tmem_ld32(lane_base + scol + 32 * c, v);
+        tc::tmem_ld_wait();
+#pragma unroll
+        for (int e = 0; e < 32; ++e)
+          if (full || s0 + 32 * c + e <= mypos) mx = fmaxf(mx, __uint_as_float(v[e]));
+      }
+      const float mt = mx * p.qscale;  // qscale > 0: the max commutes with the scale
+      float scale = 1.f;
+      const bool raise = (m == -INFINITY) ? (mt != -INFINITY) : (mt > m + kStaleMax);
+      if (raise) {
+        scale = (m == -INFINITY) ? 0.f : ex2(m - mt);
+        m = mt;
+      }
+      float sum = 0.f;
+#pragma unroll
+      for (int c = 0; c < kPN / 32; ++c) {
+        uint32_t v[32], w[16];
+        tc::tmem_ld32(lane_base + scol + 32 * c, v);
+        tc::tmem_ld_wait();
+#pragma unroll
+        for (int e = 0; e < 32; e += 2) {
+          float p0 = 0.f, p1 = 0.f;
+          if (m != -INFINITY) {
+            if (full || s0 + 32 * c + e <= mypos) p0 = ex2(fmaf(__uint_as_float(v[e]), p.qscale, -m));
+            if (full || s0 + 32 * c + e + 1 <= mypos)
+              p1 = ex2(fmaf(__uint_as_float(v[e + 1]), p.qscale, -m));
+          }
+          sum += p0 + p1;
+          const __nv_bfloat162 h = __floats2bfloat162_rn(p0, p1);
+          w[e / 2] = *reinterpret_cast<const uint32_t*>(&h);
+        }
+        // P over the S columns already read: packed pairs, columns 16c .. 16c+15
+        tc::tmem_st16(lane_base + scol + 16 * c, w);
+      }
+      l = l * scale + sum;
+      if (__any_sync(0xFFFFFFFFu, raise && j > 0)) {
+        // a row's max grew past the headroom: rescale O (every lane of the
+        // warp takes part; rows that did not raise their max scale by 1)
+        // once P V of the previous tile has landed in it
+        if (!(raise && j > 0)) scale = 1.f;
+        ok = __all_sync(0xFFFFFFFFu, mbar_wait(&odone[i], (j - 1) & 1));
+        if (!ok) break;
+        tc::fence_after_sync();
+#pragma unroll
+        for (int c = 0; c < HD / 32; ++c) {
+          uint32_t v[32];
+          tc::tmem_ld32(lane_base + ocol + 32 * c, v);
+          tc::tmem_ld_wait();
+          uint32_t w0[16], w1[16];
+#pragma unroll
+          for (int e = 0; e < 16; ++e) {
+            w0[e] = __float_as_uint(__uint_as_float(v[e]) * scale);
+            w1[e] = __float_as_uint(__uint_as_float(v[16 + e]) * scale);
+          }
+          tc::tmem_st16(lane_base + ocol + 32 * c, w0);
+          tc::tmem_st16(lane_base + ocol + 32 * c + 16, w1);
+        }
+      }
+      tc::tmem_st_wait();
+      tc::fence_before_sync();
+      mbar_arrive(&pfull[i]);
+    }
+    if (ok && n > 0) ok = __all_sync(0xFFFFFFFFu, mbar_wait(&odone[i], (n - 1) & 1));
+    if (!ok) {
+      report(p.status, WM_ERR_TIMEOUT);
+    } else {
+      __nv_bfloat16* dst =
+          reinterpret_cast<__nv_bfloat16*>(p.out) + (((int64_t)b * p.Tq + r) * p.Hq + hq) * HD;
+      const float inv = (n > 0 && l > 0.f) ? 1.f / l : 0.f;
+      tc::fence_after_sync();
+#pragma unroll
+      for (int c = 0; c < HD / 32; ++c) {
+        uint32_t v[32];
+        if (n > 0) {  // n is the same for the whole warp group
+          tc::tmem_ld32(lane_base + ocol + 32 * c, v);
+          tc::tmem_ld_wait();
+        }
+        if (r >= p.Tq) continue;
+#pragma unroll
+        for (int e = 0; e < 32; e += 8) {
+          float f[8];
+#pragma unroll
+          for (int t = 0; t < 8; ++t) f[t] = n > 0 ? __uint_as_float(v[e + t]) * inv : 0.f;
+          uint4 u;
+          __nv_bfloat162 t0 = __floats2bfloat162_rn(f[0], f[1]);
+          __nv_bfloat162 t1 = __floats2bfloat162_rn(f[2], f[3]);
+          __nv_bfloat162 t2 = __floats2bfloat162_rn(f[4], f[5]);
+          __nv_bfloat162 t3 = __floats2bfloat162_rn(f[6], f[7]);
+          u.x = *reinterpret_cast<uint32_t*>(&t0);
+          u.y = *reinterpret_cast<uint32_t*>(&t1);
+          u.z = *reinterpret_cast<uint32_t*>(&t2);
+          u.w = *reinterpret_cast<uint32_t*>(&t3);
+          *reinterpret_cast<uint4*>(dst + 32 * c + e) = u;
+        }
+      }
     }
   }
   // Every MMA this CTA issued has completed (each was waited on through its
@@ -307,7 +399,7 @@ __global__ void __launch_bounds__(kPThreads, 1)
   __syncthreads();
   if (warp == 0) {
     tc::fence_after_sync();
-    tc::tmem_dealloc(tmem, kPTmemCols);
+    tc::tmem_dealloc(tmem, kTmemCols);
   }
 }
 
@@ -323,7 +415,7 @@ cudaError_t launch_hd(const CUtensorMap& q, const CUtensorMap& k, const CUtensor
     attr_set = true;
   }
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3((p.Tq + kPM - 1) / kPM, p.Hq, p.B);
+  cfg.gridDim = dim3((p.Tq + kQT * kPM - 1) / (kQT * kPM), p.Hq, p.B);
   cfg.blockDim = dim3(kPThreads);
   cfg.dynamicSmemBytes = PShape<HD>::SMEM;
   cfg.stream = s;

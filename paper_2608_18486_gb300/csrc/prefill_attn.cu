@@ -291,16 +291,24 @@ __global__ void __launch_bounds__(kPThreads, 1)
       if (!ok) break;
       tc::fence_after_sync();
       const int s0 = j * kPN;
-      const bool full = s0 + kPN - 1 <= mypos;  // every slot of the tile is visible
+      // Visible slots of this row in the tile: e < vis (all 128 unless the
+      // diagonal crosses the tile).  The masked path only runs there.
+      const int vis = min(max(mypos - s0 + 1, 0), kPN);
       float mx = -INFINITY;
 #pragma unroll
       for (int c = 0; c < kPN / 32; ++c) {
         uint32_t v[32];
         tc::tmem_ld32(lane_base + scol + 32 * c, v);
         tc::tmem_ld_wait();
+        if (vis == kPN) {
 #pragma unroll
-        for (int e = 0; e < 32; ++e)
-          if (full || s0 + 32 * c + e <= mypos) mx = fmaxf(mx, __uint_as_float(v[e]));
+          for (int e = 0; e < 32; ++e) mx = fmaxf(mx, __uint_as_float(v[e]));
+        } else {
+          const int lim = vis - 32 * c;
+#pragma unroll
+          for (int e = 0; e < 32; ++e)
+            if (e < lim) mx = fmaxf(mx, __uint_as_float(v[e]));
+        }
       }
       const float mt = mx * p.qscale;  // qscale > 0: the max commutes with the scale
       float scale = 1.f;
@@ -309,27 +317,42 @@ __global__ void __launch_bounds__(kPThreads, 1)
         scale = (m == -INFINITY) ? 0.f : ex2(m - mt);
         m = mt;
       }
-      float sum = 0.f;
+      // p = 2^(s * qscale - m) in pairs; masked slots (and rows with nothing
+      // visible yet) give 0
+      const float2 qs2 = make_float2(p.qscale, p.qscale), nm2 = make_float2(-m, -m);
+      const bool live = m != -INFINITY;
+      float2 sum2 = make_float2(0.f, 0.f);
 #pragma unroll
       for (int c = 0; c < kPN / 32; ++c) {
         uint32_t v[32], w[16];
         tc::tmem_ld32(lane_base + scol + 32 * c, v);
         tc::tmem_ld_wait();
+        const int lim = live ? vis - 32 * c : 0;
+        if (lim >= 32) {
 #pragma unroll
-        for (int e = 0; e < 32; e += 2) {
-          float p0 = 0.f, p1 = 0.f;
-          if (m != -INFINITY) {
-            if (full || s0 + 32 * c + e <= mypos) p0 = ex2(fmaf(__uint_as_float(v[e]), p.qscale, -m));
-            if (full || s0 + 32 * c + e + 1 <= mypos)
-              p1 = ex2(fmaf(__uint_as_float(v[e + 1]), p.qscale, -m));
+          for (int e = 0; e < 32; e += 2) {
+            const float2 x = __ffma2_rn(
+                make_float2(__uint_as_float(v[e]), __uint_as_float(v[e + 1])), qs2, nm2);
+            const float2 pr = make_float2(ex2(x.x), ex2(x.y));
+            sum2 = __fadd2_rn(sum2, pr);
+            const __nv_bfloat162 h = __floats2bfloat162_rn(pr.x, pr.y);
+            w[e / 2] = *reinterpret_cast<const uint32_t*>(&h);
           }
-          sum += p0 + p1;
-          const __nv_bfloat162 h = __floats2bfloat162_rn(p0, p1);
-          w[e / 2] = *reinterpret_cast<const uint32_t*>(&h);
+        } else {
+#pragma unroll
+          for (int e = 0; e < 32; e += 2) {
+            const float2 x = __ffma2_rn(
+                make_float2(__uint_as_float(v[e]), __uint_as_float(v[e + 1])), qs2, nm2);
+            const float2 pr = make_float2(e < lim ? ex2(x.x) : 0.f, e + 1 < lim ? ex2(x.y) : 0.f);
+            sum2 = __fadd2_rn(sum2, pr);
+            const __nv_bfloat162 h = __floats2bfloat162_rn(pr.x, pr.y);
+            w[e / 2] = *reinterpret_cast<const uint32_t*>(&h);
+          }
         }
         // P over the S columns already read: packed pairs, columns 16c .. 16c+15
         tc::tmem_st16(lane_base + scol + 16 * c, w);
       }
+      const float sum = sum2.x + sum2.y;
       l = l * scale + sum;
       if (__any_sync(0xFFFFFFFFu, raise && j > 0)) {
         // a row's max grew past the headroom: rescale O (every lane of the

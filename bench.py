@@ -622,6 +622,77 @@ def run_prefill(args, w):
     print(json.dumps(line), flush=True)
 
 
+def run_pool(args, w):
+    """The cross-layer KV pool (Sec. 3.1 Steps 1-2) over the B tokens of one
+    batched evaluation: a prefill group of Sec. 3.3 hands the pool |G_q| x
+    sequences tokens at once, and at that size the router and projection are
+    real tensor-core GEMMs.  Prints one JSON line: pooled tokens/s and the
+    contraction FLOP/s (router + K/V projections) against the measured bf16
+    tensor peak."""
+    import torch
+    from paper_2608_18486_gb300 import make_config
+    from paper_2608_18486_gb300.session import DecodeSession
+    from wm_synth.device_problem import DeviceProblem
+    from wm_synth.inputs import make_problem
+
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    prob = make_problem(w, seed=0)
+    cfg = make_config(w.L, w.k, w.D, w.Hq, w.Hkv, w.d, w.p, w.page, w.dtype, w.chan_of_layer(),
+                      w.eps_rms, w.eps_qk, w.rope_theta)
+    sess = DecodeSession(cfg, w.B, prob.num_pages, prob.max_pages, dev)
+    dp = DeviceProblem(prob, sess.k_pool, sess.v_pool, dev)
+    sess.set_weights(*dp.weights())
+    stream = torch.cuda.Stream(dev)
+
+    def step():
+        sess.kv_mix(dp.h, dp.page_table, dp.slot, stream=stream)
+
+    with torch.cuda.stream(stream):
+        for _ in range(args.warmup):
+            step()
+    torch.cuda.synchronize()
+    if sess.read_status() != 0:
+        raise RuntimeError("device status set during warm-up")
+    K = args.steps
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=stream):
+        for _ in range(K):
+            step()
+    with torch.cuda.stream(stream):
+        graph.replay()
+    torch.cuda.synchronize()
+    sampler = ClockSampler(gpu_uuid_of(dev, "0"))
+    time.sleep(0.3)
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t0 = time.time()
+    with torch.cuda.stream(stream):
+        start.record(stream)
+        graph.replay()
+        end.record(stream)
+    torch.cuda.synchronize()
+    t1 = time.time()
+    clocks = sampler.stop(t0, t1)
+    if sess.read_status() != 0:
+        raise RuntimeError("device status set during the timed region")
+    ms = start.elapsed_time(end) / K
+    # two branches: router kL x L'D and k projections of Hkv*d x D, 2 FLOP per MAC
+    flops = 2.0 * 2.0 * w.B * (w.k * w.L * w.Lp * w.D + w.k * w.Hkv * w.d * w.D)
+    tflops = flops / (ms * 1e-3) / 1e12
+    peaks = json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
+    peak = float(peaks["bf16_tflops_sustained"])
+    from wm_synth import configs as wcfg
+    line = {"metric": "batched pool tokens/s (router + K/V projections + cache write, one evaluation)",
+            "value": w.B / (ms * 1e-3), "unit": "tokens/s", "n_gpus": 1, "steps": K,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "dtype": w.dtype,
+            "data": "synthetic", "config": dict(config_dict(w, 1), mode="pool", tokens=w.B),
+            "roofline": {"bound": "tensor", "achieved": tflops, "peak": peak, "unit": "TFLOP/s",
+                         "frac": tflops / peak, "peak_kind": "measured sustained bf16",
+                         "flops_per_step": flops, "bytes_per_step": wcfg.mix_bytes(w)},
+            "clocks": clocks}
+    print(json.dumps(line), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -629,9 +700,10 @@ def main():
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
-    ap.add_argument("--mode", default="path", choices=["path", "model", "prefill"],
+    ap.add_argument("--mode", default="path", choices=["path", "model", "prefill", "pool"],
                     help="path: the WhiteMatter decode hot path (default); model: a whole-model "
-                         "decode step; prefill: causal channel attention of a prefill pass")
+                         "decode step; prefill: causal channel attention of a prefill pass; "
+                         "pool: one batched pool evaluation over B tokens")
     ap.add_argument("--groups", type=int, default=8,
                     help="--mode prefill: strided Gauss-Seidel groups (1: a Jacobi pass)")
     ap.add_argument("--intermediate", type=int, default=0,
@@ -657,6 +729,8 @@ def main():
         run_model(args, w)
     elif args.mode == "prefill":
         run_prefill(args, w)
+    elif args.mode == "pool":
+        run_pool(args, w)
     else:
         run_gpu(args, w)
 

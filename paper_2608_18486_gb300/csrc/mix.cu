@@ -29,6 +29,11 @@ namespace {
 constexpr int kMixThreads = 256;
 constexpr int kChanGroup = 4; // channels mixed per CTA
 constexpr int kVecPerThread = 2;  // 8-element vectors per thread: D <= 256*8*2
+// Token counts from which the pool runs its batched forms of prenorm and mix
+// (prefill groups): several tokens per CTA, whole warps on every row.  Below
+// it (decode steps) one token per CTA spreads the few tokens over more SMs.
+constexpr int kBatchedTokens = 64;
+constexpr int kMixCG = 8;     // channels per CTA in the batched mix
 
 __device__ __forceinline__ void pdl_wait() {
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
@@ -120,6 +125,58 @@ __global__ void __launch_bounds__(kMixThreads) prenorm_kernel(const MixParams p)
     const int s = p.slot[b];
     const double pos = (double)(s - 1);
     for (int i = tid; i < p.d / 2; i += kMixThreads) {
+      const double a = pos * p.inv_freq[i];
+      const double two_pi = 6.283185307179586476925286766559;
+      const float ar = (float)(a - two_pi * rint(a / two_pi));
+      float sn, cs;
+      sincosf(ar, &sn, &cs);
+      p.rope_cs[((int64_t)b * (p.d / 2) + i) * 2] = cs;
+      p.rope_cs[((int64_t)b * (p.d / 2) + i) * 2 + 1] = sn;
+    }
+  }
+}
+
+// Batched form: one warp per (token, layer) row, 8 rows per CTA, 16-byte
+// vectors.  Same outputs as prenorm_kernel.
+template <typename T>
+__global__ void __launch_bounds__(kMixThreads) prenorm_rows_kernel(const MixParams p) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int row = blockIdx.x * (kMixThreads / 32) + warp;  // b * L + l
+  pdl_wait();
+  if (row >= p.B * p.L) return;  // warp-level from here on
+  const int b = row / p.L, l = row % p.L;
+  const int nvec = p.D / 8;
+  const T* hp = reinterpret_cast<const T*>(p.h) + (int64_t)row * p.D;
+  float ss = 0.f;
+  for (int v = lane; v < nvec; v += 32) {
+    float f[8];
+    load8f<T>(hp + v * 8, f);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) ss = fmaf(f[i], f[i], ss);
+  }
+  const float r = rsqrtf(warp_sum(ss) / (float)p.D + p.eps_rms);
+  if (lane == 0) p.inv_rms[row] = r;
+  const int from_top = p.L - 1 - l;
+  if (from_top % p.p == 0) {  // router input block m holds layer L-1-m*p
+    const int m = from_top / p.p;
+    for (int X = 0; X < 2; ++X) {
+      const T* g = reinterpret_cast<const T*>(p.pre_g[X]);
+      T* xo = reinterpret_cast<T*>(p.xi) + ((int64_t)X * p.B + b) * ((int64_t)p.Lp * p.D) +
+              (int64_t)m * p.D;
+      for (int v = lane; v < nvec; v += 32) {
+        float f[8], gv[8];
+        load8f<T>(hp + v * 8, f);
+        load8f<T>(g + v * 8, gv);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) f[i] *= r * gv[i];
+        store8f<T>(xo + v * 8, f);
+      }
+    }
+  }
+  if (l == 0) {
+    // RoPE angle pos * theta^(-2i/d) in fp64, reduced to [-pi, pi] before sincosf
+    const double pos = (double)(p.slot[b] - 1);
+    for (int i = lane; i < p.d / 2; i += 32) {
       const double a = pos * p.inv_freq[i];
       const double two_pi = 6.283185307179586476925286766559;
       const float ar = (float)(a - two_pi * rint(a / two_pi));
@@ -329,6 +386,117 @@ __global__ void __launch_bounds__(kMixThreads) mix_kernel(const MixParams p) {
   }
 }
 
+// Batched form: one CTA per (tb tokens, branch, kMixCG channels); tpt
+// threads (whole warps) per token, thread u of a token owning the 8-element
+// vectors u, u + tpt, ... of D.  alpha of the CTA's tokens is summed from the
+// router's split partials once, into shared memory.
+template <typename T, int VPT>
+__global__ void __launch_bounds__(kMixThreads) mix_tokens_kernel(const MixParams p, int tpt, int tb) {
+  extern __shared__ float sm[];  // alpha[tb][kMixCG][L], rl[tb][L], red[warps][kMixCG]
+  const int X = blockIdx.y, j0 = blockIdx.z * kMixCG;
+  const int nj = min(kMixCG, p.k - j0);
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int t = tid / tpt, u = tid % tpt;
+  const int b0 = blockIdx.x * tb, b = b0 + t;
+  const bool live = t < tb && b < p.B;
+  const int L = p.L, kL = p.k * p.L, nvec = p.D / 8;
+  float* alpha = sm;
+  float* rl = alpha + tb * kMixCG * L;
+  float* red = rl + tb * L;
+  pdl_wait();
+  const T* br = reinterpret_cast<const T*>(p.br[X]);
+  for (int i = tid; i < tb * nj * L; i += blockDim.x) {
+    const int tt = i / (nj * L), rem = i % (nj * L);
+    const int bb = b0 + tt, o = j0 * L + rem;
+    float z = 0.f;
+    if (bb < p.B) {
+      z = ldf(br + o);
+      const float* zp = p.zpart + ((int64_t)X * p.nsplit_r * p.B + bb) * kL + o;
+      for (int s2 = 0; s2 < p.nsplit_r; ++s2) z += zp[(int64_t)s2 * p.B * kL];
+    }
+    alpha[tt * kMixCG * L + rem] = z;  // [tt][jj][l] with jj = rem / L, l = rem % L
+  }
+  for (int i = tid; i < tb * L; i += blockDim.x) {
+    const int bb = b0 + i / L;
+    rl[i] = bb < p.B ? p.inv_rms[(int64_t)bb * L + i % L] : 0.f;
+  }
+  __syncthreads();
+
+  const T* hp = reinterpret_cast<const T*>(p.h) + (int64_t)b * L * p.D;
+  const T* g = reinterpret_cast<const T*>(p.pre_g[X]);
+  float gv[VPT][8];
+  float acc[kMixCG][VPT][8];
+#pragma unroll
+  for (int v = 0; v < VPT; ++v) {
+    const int vi = u + v * tpt;
+    if (live && vi < nvec) load8f<T>(g + vi * 8, gv[v]);
+#pragma unroll
+    for (int jj = 0; jj < kMixCG; ++jj)
+#pragma unroll
+      for (int i = 0; i < 8; ++i) acc[jj][v][i] = 0.f;
+  }
+  if (live) {
+    const float* al = alpha + t * kMixCG * L;
+#pragma unroll 2
+    for (int l = 0; l < L; ++l) {
+      const float r = rl[t * L + l];
+      float a[kMixCG];
+#pragma unroll
+      for (int jj = 0; jj < kMixCG; ++jj) a[jj] = jj < nj ? al[jj * L + l] : 0.f;
+#pragma unroll
+      for (int v = 0; v < VPT; ++v) {
+        const int vi = u + v * tpt;
+        if (vi < nvec) {
+          float hv[8];
+          load8f<T>(hp + (int64_t)l * p.D + vi * 8, hv);
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            const float hh = hv[i] * r * gv[v][i];  // pre-mix RMSNorm with gain
+#pragma unroll
+            for (int jj = 0; jj < kMixCG; ++jj) acc[jj][v][i] = fmaf(a[jj], hh, acc[jj][v][i]);
+          }
+        }
+      }
+    }
+  }
+  // per-channel sums of squares over the token's warps
+#pragma unroll
+  for (int jj = 0; jj < kMixCG; ++jj) {
+    float q = 0.f;
+#pragma unroll
+    for (int v = 0; v < VPT; ++v)
+#pragma unroll
+      for (int i = 0; i < 8; ++i) q = fmaf(acc[jj][v][i], acc[jj][v][i], q);
+    q = warp_sum(q);
+    if (lane == 0) red[warp * kMixCG + jj] = q;
+  }
+  __syncthreads();
+  if (!live) return;
+  const int w0 = t * (tpt / 32), nw = tpt / 32;
+  T* xop = reinterpret_cast<T*>(p.xop);
+#pragma unroll
+  for (int jj = 0; jj < kMixCG; ++jj) {
+    if (jj >= nj) break;
+    float q = 0.f;
+    for (int w = 0; w < nw; ++w) q += red[(w0 + w) * kMixCG + jj];
+    const float sc = rsqrtf(q / (float)p.D + p.eps_rms);
+    const int j = j0 + jj;
+    const T* cg = reinterpret_cast<const T*>(p.ch_g[X]) + (int64_t)j * p.D;
+    T* xo = xop + (((int64_t)X * p.k + j) * p.B + b) * p.D;
+#pragma unroll
+    for (int v = 0; v < VPT; ++v) {
+      const int vi = u + v * tpt;
+      if (vi < nvec) {
+        float cv[8], o[8];
+        load8f<T>(cg + vi * 8, cv);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) o[i] = acc[jj][v][i] * sc * cv[i];
+        store8f<T>(xo + vi * 8, o);
+      }
+    }
+  }
+}
+
 // ---------------------------------------------------------------- epilogue
 // fp32 path: one CTA per (token, channel, branch), a warp per kv head; lane t
 // handles the RoPE pairs (i, i + HD/2) for i = t, t + 32, ...
@@ -396,7 +564,15 @@ template <typename T>
 cudaError_t launch_all(MixParams& p, cudaStream_t s) {
   const int kL = p.k * p.L;
   const bool bf16 = sizeof(T) == 2;
-  cudaError_t e = launch_pdl(prenorm_kernel<T>, dim3(p.L, p.B), dim3(kMixThreads), 0, s, p);
+  const bool batched = p.B >= kBatchedTokens;
+  cudaError_t e;
+  if (batched) {
+    const int rows = p.B * p.L, per = kMixThreads / 32;
+    e = launch_pdl(prenorm_rows_kernel<T>, dim3((rows + per - 1) / per), dim3(kMixThreads), 0, s,
+                   p);
+  } else {
+    e = launch_pdl(prenorm_kernel<T>, dim3(p.L, p.B), dim3(kMixThreads), 0, s, p);
+  }
   if (e != cudaSuccess) return e;
   if (bf16 && router_tc_supported(p.B)) {
     e = launch_router_tc(p, s);
@@ -418,7 +594,19 @@ cudaError_t launch_all(MixParams& p, cudaStream_t s) {
     e = launch_pdl(gemm_wxT_simt<T, T>, grid, dim3(256), 0, s, a);
   }
   if (e != cudaSuccess) return e;
-  {
+  if (batched) {
+    const int nvec = p.D / 8;
+    const bool two = nvec > kMixThreads;  // D > 2048: two vectors per thread
+    const int per = two ? (nvec + 1) / 2 : nvec;
+    const int tpt = (per + 31) / 32 * 32;
+    const int tb = tpt >= kMixThreads ? 1 : kMixThreads / tpt;
+    const size_t smem = sizeof(float) * ((size_t)tb * kMixCG * p.L + (size_t)tb * p.L +
+                                         (size_t)(tb * tpt / 32) * kMixCG);
+    dim3 grid((p.B + tb - 1) / tb, 2, (p.k + kMixCG - 1) / kMixCG);
+    e = two ? launch_pdl(mix_tokens_kernel<T, 2>, grid, dim3(tb * tpt), smem, s, p, tpt, tb)
+            : launch_pdl(mix_tokens_kernel<T, 1>, grid, dim3(tb * tpt), smem, s, p, tpt, tb);
+    if (e != cudaSuccess) return e;
+  } else {
     const size_t smem = sizeof(float) * (kChanGroup * p.L + p.L);
     dim3 grid(p.B, 2, (p.k + kChanGroup - 1) / kChanGroup);
     e = launch_pdl(mix_kernel<T>, grid, dim3(kMixThreads), smem, s, p);

@@ -412,6 +412,7 @@ __global__ void __launch_bounds__(kMixThreads) mix_tokens_kernel(const MixParams
     if (bb < p.B) {
       z = ldf(br + o);
       const float* zp = p.zpart + ((int64_t)X * p.nsplit_r * p.B + bb) * kL + o;
+#pragma unroll 8
       for (int s2 = 0; s2 < p.nsplit_r; ++s2) z += zp[(int64_t)s2 * p.B * kL];
     }
     alpha[tt * kMixCG * L + rem] = z;  // [tt][jj][l] with jj = rem / L, l = rem % L

@@ -204,48 +204,74 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     qg1[t] = i < HALF ? __bfloat162float(p.qk_g[(int64_t)j * HD + i + HALF]) : 0.f;
   }
   const float* cs_tab = p.rope_smem_off > 0 ? rope_s : p.rope_cs;
-  for (int it = warp; it < nb * HPT; it += kTcThreads / 32) {
-    const int n = it / HPT, hl = it % HPT;  // n: token within the tile
-    const int hh = mt * HPT + hl;
-    if (hh >= p.Hkv) continue;
-    const int s = s_slot[n], pg = s_page[n];
-    if (pg < 0) {
-      if (reporter && hl == 0 && lane == 0) report(p.status, WM_ERR_BOUNDS);
-      continue;
-    }
-    const float* src = T + n * kTcM + hl * HD;
-    float y0[NP], y1[NP];
+  // Each warp takes IPW items per round, their loads, reductions and stores
+  // interleaved so that the latencies overlap.
+  constexpr int IPW = 4;
+  constexpr int NW = kTcThreads / 32;
+  const int nitems = nb * HPT;
+  for (int it0 = warp * IPW; it0 < nitems; it0 += NW * IPW) {
+    float y0[IPW][NP], y1[IPW][NP];
+    int n_[IPW], hh_[IPW], pg_[IPW];
+    bool on[IPW];
 #pragma unroll
-    for (int t = 0; t < NP; ++t) {
-      const int i = lane + 32 * t;
-      y0[t] = i < HALF ? src[i] : 0.f;
-      y1[t] = i < HALF ? src[i + HALF] : 0.f;
+    for (int q = 0; q < IPW; ++q) {
+      const int it = it0 + q;
+      const int n = it / HPT, hl = it % HPT;  // n: token within the tile
+      n_[q] = n;
+      hh_[q] = mt * HPT + hl;
+      pg_[q] = it < nitems ? s_page[n] : -1;
+      on[q] = it < nitems && hh_[q] < p.Hkv && pg_[q] >= 0;
+      if (it < nitems && hh_[q] < p.Hkv && pg_[q] < 0 && reporter && hl == 0 && lane == 0)
+        report(p.status, WM_ERR_BOUNDS);
+      const float* src = T + n * kTcM + hl * HD;
+#pragma unroll
+      for (int t = 0; t < NP; ++t) {
+        const int i = lane + 32 * t;
+        y0[q][t] = on[q] && i < HALF ? src[i] : 0.f;
+        y1[q][t] = on[q] && i < HALF ? src[i + HALF] : 0.f;
+      }
     }
     if (X == 0) {
-      float ss = 0.f;
+      float ss[IPW];
 #pragma unroll
-      for (int t = 0; t < NP; ++t) ss = fmaf(y0[t], y0[t], fmaf(y1[t], y1[t], ss));
-      ss = warp_sum(ss);
-      const float rr = rsqrtf(ss / (float)HD + p.eps_qk);
+      for (int q = 0; q < IPW; ++q) {
+        ss[q] = 0.f;
+#pragma unroll
+        for (int t = 0; t < NP; ++t) ss[q] = fmaf(y0[q][t], y0[q][t], fmaf(y1[q][t], y1[q][t], ss[q]));
+      }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1)
+#pragma unroll
+        for (int q = 0; q < IPW; ++q) ss[q] += __shfl_xor_sync(0xFFFFFFFFu, ss[q], o);
+#pragma unroll
+      for (int q = 0; q < IPW; ++q) {
+        const float rr = rsqrtf(ss[q] / (float)HD + p.eps_qk);
+        const int row = cs_tab == rope_s ? n_[q] : n0 + n_[q];
+#pragma unroll
+        for (int t = 0; t < NP; ++t) {
+          const int i = lane + 32 * t;
+          if (on[q] && i < HALF) {
+            const float x0 = y0[q][t] * rr * qg0[t], x1 = y1[q][t] * rr * qg1[t];
+            const float2 csn = reinterpret_cast<const float2*>(cs_tab)[row * HALF + i];
+            y0[q][t] = x0 * csn.x - x1 * csn.y;  // rotate-half RoPE
+            y1[q][t] = x1 * csn.x + x0 * csn.y;
+          }
+        }
+      }
+    }
+#pragma unroll
+    for (int q = 0; q < IPW; ++q) {
+      if (!on[q]) continue;
+      const int s = s_slot[n_[q]];
+      __nv_bfloat16* dst =
+          pool + ((((int64_t)j * p.num_pages + pg_[q]) * p.Hkv + hh_[q]) * p.P + (s & (p.P - 1))) * HD;
 #pragma unroll
       for (int t = 0; t < NP; ++t) {
         const int i = lane + 32 * t;
         if (i < HALF) {
-          const float x0 = y0[t] * rr * qg0[t], x1 = y1[t] * rr * qg1[t];
-          const float2 csn = reinterpret_cast<const float2*>(cs_tab)[(cs_tab == rope_s ? n : n0 + n) * HALF + i];
-          y0[t] = x0 * csn.x - x1 * csn.y;  // rotate-half RoPE
-          y1[t] = x1 * csn.x + x0 * csn.y;
+          dst[i] = __float2bfloat16_rn(y0[q][t]);
+          dst[i + HALF] = __float2bfloat16_rn(y1[q][t]);
         }
-      }
-    }
-    __nv_bfloat16* dst =
-        pool + ((((int64_t)j * p.num_pages + pg) * p.Hkv + hh) * p.P + (s & (p.P - 1))) * HD;
-#pragma unroll
-    for (int t = 0; t < NP; ++t) {
-      const int i = lane + 32 * t;
-      if (i < HALF) {
-        dst[i] = __float2bfloat16_rn(y0[t]);
-        dst[i + HALF] = __float2bfloat16_rn(y1[t]);
       }
     }
   }

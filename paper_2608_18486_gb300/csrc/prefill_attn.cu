@@ -49,10 +49,14 @@ constexpr float kStaleMax = 8.f;            // log2 headroom before O is rescale
 template <int HD>
 struct PShape {
   static constexpr int CB = (HD + 63) / 64;          // 64-column blocks of a head row
-  static constexpr int NST = HD <= 64 ? 3 : 2;       // depth of the K and V rings
+  // Ring depths: the next K tile is waited for first (S of the next KV tile
+  // is issued behind P V of this one), so K gets the deeper ring.
+  static constexpr int NSK = HD <= 64 ? 4 : 3;
+  static constexpr int NSV = HD <= 64 ? 4 : 2;
   static constexpr uint32_t Q_BYTES = CB * kBlock;   // one Q tile
   static constexpr uint32_t KV_BYTES = CB * kBlock;  // one K or V tile
-  static constexpr uint32_t SMEM = kQT * Q_BYTES + 2 * NST * KV_BYTES + 1024;  // + alignment
+  static constexpr uint32_t SMEM = kQT * Q_BYTES + (NSK + NSV) * KV_BYTES + 1024;  // + alignment
+  static_assert(SMEM <= 227 * 1024, "shared memory");
 };
 
 struct PrefillParams {
@@ -76,9 +80,9 @@ __global__ void __launch_bounds__(kPThreads, 1)
                         const __grid_constant__ CUtensorMap tmK,
                         const __grid_constant__ CUtensorMap tmV, const PrefillParams p) {
   using SH = PShape<HD>;
-  constexpr int CB = SH::CB, NST = SH::NST;
+  constexpr int CB = SH::CB, NSK = SH::NSK, NSV = SH::NSV;
   extern __shared__ uint8_t smem_dyn[];
-  __shared__ uint64_t qbar, kfull[NST], kempty[NST], vfull[NST], vempty[NST];
+  __shared__ uint64_t qbar, kfull[NSK], kempty[NSK], vfull[NSV], vempty[NSV];
   __shared__ uint64_t sfull[kQT], pfull[kQT], odone[kQT];
   __shared__ uint32_t tmem_base;
   __shared__ int wmax[kSoftWarps];
@@ -90,14 +94,16 @@ __global__ void __launch_bounds__(kPThreads, 1)
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_dyn) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
   uint8_t* Qs = base;                         // [kQT] Q tiles
-  uint8_t* Ks = Qs + kQT * SH::Q_BYTES;       // [NST] K tiles
-  uint8_t* Vs = Ks + NST * SH::KV_BYTES;      // [NST] V tiles
+  uint8_t* Ks = Qs + kQT * SH::Q_BYTES;       // [NSK] K tiles
+  uint8_t* Vs = Ks + NSK * SH::KV_BYTES;      // [NSV] V tiles
 
   if (tid == 0) {
     mbar_init(&qbar, 1);
-    for (int s = 0; s < NST; ++s) {
+    for (int s = 0; s < NSK; ++s) {
       mbar_init(&kfull[s], 1);
       mbar_init(&kempty[s], 1);
+    }
+    for (int s = 0; s < NSV; ++s) {
       mbar_init(&vfull[s], 1);
       mbar_init(&vempty[s], 1);
     }
@@ -154,46 +160,57 @@ __global__ void __launch_bounds__(kPThreads, 1)
 
   if (warp == kLoadWarp) {
     // ================================================================ TMA
-    if (lane == 0 && nmax > 0) {
+    // Lane t owns box t of every KV tile (one box per page, or one per 128
+    // slots of a longer page): its page id for the next tile is fetched
+    // while the current tile is issued, so no page-table load sits on the
+    // issue path.  Lane 0 posts the expected bytes before the lanes copy.
+    if (nmax > 0) {
       bool ok = true;
-      mbar_arrive_expect_tx(&qbar, kQT * SH::Q_BYTES);
-      for (int i = 0; i < kQT; ++i)
-#pragma unroll
-        for (int cb = 0; cb < CB; ++cb)
-          tc::tma_load_2d(Qs + i * SH::Q_BYTES + cb * kBlock, &tmQ, hq * HD + cb * 64,
-                          b * p.Tq + r0 + i * kPM, &qbar);
-      const int boxes = p.P >= kPN ? 1 : kPN >> p.log2P;
-      const int brows = p.P >= kPN ? kPN : p.P;
-      auto load_tile = [&](const CUtensorMap* tm, uint8_t* dst, int j, uint64_t* bar) {
-        mbar_arrive_expect_tx(bar, SH::KV_BYTES);
-        const int s0 = j * kPN;
-        for (int t = 0; t < boxes; ++t) {
-          const int s = s0 + t * brows;  // first slot of the box
-          const int lp = s >> p.log2P;   // logical page
-          int row = -brows;              // fully outside the map: reads zeros
-          if (s <= tmaxpos && lp < p.max_pages) {
-            const int pg = p.page_table[(int64_t)b * p.max_pages + lp];
-            if (pg >= 0 && pg < p.num_pages)
-              row = (int)((((int64_t)p.chan * p.num_pages + pg) * p.Hkv + hkv) * p.P +
-                          (s & (p.P - 1)));
-            else
-              report(p.status, WM_ERR_BOUNDS);
-          }
+      if (lane == 0) {
+        mbar_arrive_expect_tx(&qbar, kQT * SH::Q_BYTES);
+        for (int i = 0; i < kQT; ++i)
 #pragma unroll
           for (int cb = 0; cb < CB; ++cb)
-            tc::tma_load_2d(dst + cb * kBlock + t * brows * 128, tm, cb * 64, row, bar);
-        }
-      };
-      for (int j = 0; j < nmax && ok; ++j) {
-        const int st = j % NST, use = j / NST;
-        if (j >= NST) ok = mbar_wait(&kempty[st], (use - 1) & 1);
-        if (!ok) break;
-        load_tile(&tmK, Ks + st * SH::KV_BYTES, j, &kfull[st]);
-        if (j >= NST) ok = mbar_wait(&vempty[st], (use - 1) & 1);
-        if (!ok) break;
-        load_tile(&tmV, Vs + st * SH::KV_BYTES, j, &vfull[st]);
+            tc::tma_load_2d(Qs + i * SH::Q_BYTES + cb * kBlock, &tmQ, hq * HD + cb * 64,
+                            b * p.Tq + r0 + i * kPM, &qbar);
       }
-      if (!ok) report(p.status, WM_ERR_TIMEOUT);
+      const int boxes = p.P >= kPN ? 1 : kPN >> p.log2P;  // <= 16 for pages of >= 8 slots
+      const int brows = p.P >= kPN ? kPN : p.P;
+      // tensor-map row of this lane's box of KV tile j (-brows: read zeros)
+      auto box_row = [&](int j) -> int {
+        const int s = j * kPN + lane * brows;  // first slot of the box
+        const int lp = s >> p.log2P;           // logical page
+        int row = -brows;
+        if (lane < boxes && s <= tmaxpos && lp < p.max_pages) {
+          const int pg = p.page_table[(int64_t)b * p.max_pages + lp];
+          if (pg >= 0 && pg < p.num_pages)
+            row = (int)((((int64_t)p.chan * p.num_pages + pg) * p.Hkv + hkv) * p.P + (s & (p.P - 1)));
+          else
+            report(p.status, WM_ERR_BOUNDS);
+        }
+        return row;
+      };
+      auto load_tile = [&](const CUtensorMap* tm, uint8_t* dst, int row, uint64_t* bar) {
+        if (lane == 0) mbar_arrive_expect_tx(bar, SH::KV_BYTES);
+        __syncwarp();
+        if (lane < boxes)
+#pragma unroll
+          for (int cb = 0; cb < CB; ++cb)
+            tc::tma_load_2d(dst + cb * kBlock + lane * brows * 128, tm, cb * 64, row, bar);
+      };
+      int row_next = box_row(0);
+      for (int j = 0; j < nmax && ok; ++j) {
+        const int row = row_next;
+        if (j + 1 < nmax) row_next = box_row(j + 1);
+        const int sk = j % NSK, sv = j % NSV;
+        if (j >= NSK) ok = __all_sync(0xFFFFFFFFu, mbar_wait(&kempty[sk], (j / NSK - 1) & 1));
+        if (!ok) break;
+        load_tile(&tmK, Ks + sk * SH::KV_BYTES, row, &kfull[sk]);
+        if (j >= NSV) ok = __all_sync(0xFFFFFFFFu, mbar_wait(&vempty[sv], (j / NSV - 1) & 1));
+        if (!ok) break;
+        load_tile(&tmV, Vs + sv * SH::KV_BYTES, row, &vfull[sv]);
+      }
+      if (!ok && lane == 0) report(p.status, WM_ERR_TIMEOUT);
     }
   } else if (warp == kMmaWarp) {
     // ================================================================ MMA
@@ -208,7 +225,7 @@ __global__ void __launch_bounds__(kPThreads, 1)
     auto issue_s = [&](int i, int j) {  // S_i = Q_i K_j^T
       if (lane == 0) {
         const uint32_t q0 = smem_u32(Qs + i * SH::Q_BYTES);
-        const uint32_t k0 = smem_u32(Ks + (j % NST) * SH::KV_BYTES);
+        const uint32_t k0 = smem_u32(Ks + (j % NSK) * SH::KV_BYTES);
 #pragma unroll
         for (int kk = 0; kk < HD / 16; ++kk) {
           const uint32_t off = (kk >> 2) * kBlock + (kk & 3) * 32;
@@ -220,7 +237,7 @@ __global__ void __launch_bounds__(kPThreads, 1)
     };
     auto issue_pv = [&](int i, int j) {  // O_i += P_i V_j
       if (lane == 0) {
-        const uint32_t v0 = smem_u32(Vs + (j % NST) * SH::KV_BYTES);
+        const uint32_t v0 = smem_u32(Vs + (j % NSV) * SH::KV_BYTES);
 #pragma unroll
         for (int kk = 0; kk < kPN / 16; ++kk)
           tc::mma_bf16_ts(tmem + 256 + 128 * i, tmem + 128 * i + 8 * kk,
@@ -239,8 +256,8 @@ __global__ void __launch_bounds__(kPThreads, 1)
       }
     }
     for (int j = 0; j < nmax && ok; ++j) {
-      const int st = j % NST;
-      ok = wait_all(&vfull[st], (j / NST) & 1);
+      const int st = j % NSV;
+      ok = wait_all(&vfull[st], (j / NSV) & 1);
       if (!ok) break;
       const int s0 = j * kPN;
       if (j == nmax - 1 && s0 + kPN - 1 > tmaxpos) {
@@ -258,7 +275,7 @@ __global__ void __launch_bounds__(kPThreads, 1)
       }
       const bool more = j + 1 < nmax;
       if (more) {
-        ok = wait_all(&kfull[(j + 1) % NST], ((j + 1) / NST) & 1);
+        ok = wait_all(&kfull[(j + 1) % NSK], ((j + 1) / NSK) & 1);
         if (!ok) break;
       }
       for (int i = 0; i < kQT && ok; ++i) {
@@ -271,7 +288,7 @@ __global__ void __launch_bounds__(kPThreads, 1)
       }
       if (lane == 0) {
         tc::mma_commit(&vempty[st]);
-        if (more) tc::mma_commit(&kempty[(j + 1) % NST]);
+        if (more) tc::mma_commit(&kempty[(j + 1) % NSK]);
       }
       __syncwarp();
     }
@@ -294,21 +311,23 @@ __global__ void __launch_bounds__(kPThreads, 1)
       // Visible slots of this row in the tile: e < vis (all 128 unless the
       // diagonal crosses the tile).  The masked path only runs there.
       const int vis = min(max(mypos - s0 + 1, 0), kPN);
+      // the whole S row in one TMEM read
+      uint32_t v[kPN / 32][32];
+#pragma unroll
+      for (int c = 0; c < kPN / 32; ++c) tc::tmem_ld32(lane_base + scol + 32 * c, v[c]);
+      tc::tmem_ld_wait();
       float mx = -INFINITY;
+      if (vis == kPN) {
 #pragma unroll
-      for (int c = 0; c < kPN / 32; ++c) {
-        uint32_t v[32];
-        tc::tmem_ld32(lane_base + scol + 32 * c, v);
-        tc::tmem_ld_wait();
-        if (vis == kPN) {
+        for (int c = 0; c < kPN / 32; ++c)
 #pragma unroll
-          for (int e = 0; e < 32; ++e) mx = fmaxf(mx, __uint_as_float(v[e]));
-        } else {
-          const int lim = vis - 32 * c;
+          for (int e = 0; e < 32; ++e) mx = fmaxf(mx, __uint_as_float(v[c][e]));
+      } else {
+#pragma unroll
+        for (int c = 0; c < kPN / 32; ++c)
 #pragma unroll
           for (int e = 0; e < 32; ++e)
-            if (e < lim) mx = fmaxf(mx, __uint_as_float(v[e]));
-        }
+            if (32 * c + e < vis) mx = fmaxf(mx, __uint_as_float(v[c][e]));
       }
       const float mt = mx * p.qscale;  // qscale > 0: the max commutes with the scale
       float scale = 1.f;
@@ -324,15 +343,13 @@ __global__ void __launch_bounds__(kPThreads, 1)
       float2 sum2 = make_float2(0.f, 0.f);
 #pragma unroll
       for (int c = 0; c < kPN / 32; ++c) {
-        uint32_t v[32], w[16];
-        tc::tmem_ld32(lane_base + scol + 32 * c, v);
-        tc::tmem_ld_wait();
+        uint32_t w[16];
         const int lim = live ? vis - 32 * c : 0;
         if (lim >= 32) {
 #pragma unroll
           for (int e = 0; e < 32; e += 2) {
             const float2 x = __ffma2_rn(
-                make_float2(__uint_as_float(v[e]), __uint_as_float(v[e + 1])), qs2, nm2);
+                make_float2(__uint_as_float(v[c][e]), __uint_as_float(v[c][e + 1])), qs2, nm2);
             const float2 pr = make_float2(ex2(x.x), ex2(x.y));
             sum2 = __fadd2_rn(sum2, pr);
             const __nv_bfloat162 h = __floats2bfloat162_rn(pr.x, pr.y);
@@ -342,14 +359,14 @@ __global__ void __launch_bounds__(kPThreads, 1)
 #pragma unroll
           for (int e = 0; e < 32; e += 2) {
             const float2 x = __ffma2_rn(
-                make_float2(__uint_as_float(v[e]), __uint_as_float(v[e + 1])), qs2, nm2);
+                make_float2(__uint_as_float(v[c][e]), __uint_as_float(v[c][e + 1])), qs2, nm2);
             const float2 pr = make_float2(e < lim ? ex2(x.x) : 0.f, e + 1 < lim ? ex2(x.y) : 0.f);
             sum2 = __fadd2_rn(sum2, pr);
             const __nv_bfloat162 h = __floats2bfloat162_rn(pr.x, pr.y);
             w[e / 2] = *reinterpret_cast<const uint32_t*>(&h);
           }
         }
-        // P over the S columns already read: packed pairs, columns 16c .. 16c+15
+        // P over the S columns (all read above): packed pairs, columns 16c .. 16c+15
         tc::tmem_st16(lane_base + scol + 16 * c, w);
       }
       const float sum = sum2.x + sum2.y;

@@ -34,6 +34,16 @@ constexpr int kVecPerThread = 2;  // 8-element vectors per thread: D <= 256*8*2
 // it (decode steps) one token per CTA spreads the few tokens over more SMs.
 constexpr int kBatchedTokens = 64;
 constexpr int kMixCG = 8;     // channels per CTA in the batched mix
+constexpr int kMixLC = 8;     // most layers per staged chunk of h in the batched mix
+constexpr size_t kMixStageBudget = 160 * 1024;  // shared memory for the staged chunks
+
+// 16-byte asynchronous global -> shared copies (no registers held while in flight)
+__device__ __forceinline__ void cp_async16(void* dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
 
 __device__ __forceinline__ void pdl_wait() {
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
@@ -389,10 +399,18 @@ __global__ void __launch_bounds__(kMixThreads) mix_kernel(const MixParams p) {
 // Batched form: one CTA per (tb tokens, branch, kMixCG channels); tpt
 // threads (whole warps) per token, thread u of a token owning the 8-element
 // vectors u, u + tpt, ... of D.  alpha of the CTA's tokens is summed from the
-// router's split partials once, into shared memory.
+// router's split partials once, into shared memory.  Each thread streams its
+// own vectors of h through a private 2 x kMixLC-layer buffer in shared memory
+// with asynchronous copies, so many loads are in flight without holding
+// registers.
 template <typename T, int VPT>
-__global__ void __launch_bounds__(kMixThreads) mix_tokens_kernel(const MixParams p, int tpt, int tb) {
-  extern __shared__ float sm[];  // alpha[tb][kMixCG][L], rl[tb][L], red[warps][kMixCG]
+__global__ void __launch_bounds__(kMixThreads) mix_tokens_kernel(const MixParams p, int tpt, int tb,
+                                                                  int lc) {
+  // alpha[tb][kMixCG][L], rl[tb][L], red[warps][kMixCG], then (16-byte
+  // aligned) the h staging buffers [2][lc][VPT][threads] of one vector
+  // (8 elements: VB 16-byte units) each; lc <= kMixLC layers per chunk
+  extern __shared__ float sm[];
+  constexpr int VB = 8 * (int)sizeof(T) / 16;
   const int X = blockIdx.y, j0 = blockIdx.z * kMixCG;
   const int nj = min(kMixCG, p.k - j0);
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -403,7 +421,31 @@ __global__ void __launch_bounds__(kMixThreads) mix_tokens_kernel(const MixParams
   float* alpha = sm;
   float* rl = alpha + tb * kMixCG * L;
   float* red = rl + tb * L;
+  uint4* hbuf = reinterpret_cast<uint4*>(
+      (reinterpret_cast<uintptr_t>(red + (blockDim.x / 32) * kMixCG) + 15) & ~static_cast<uintptr_t>(15));
+  const int nth = blockDim.x;
+  auto hslot = [&](int stage, int l, int v) -> uint4* {
+    return hbuf + (((stage * lc + l) * VPT + v) * nth + tid) * VB;
+  };
+  const T* hp = reinterpret_cast<const T*>(p.h) + (int64_t)b * L * p.D;
+  // copies of layers [l0, l0 + lc) of this thread's vectors into `stage`
+  auto stage_chunk = [&](int stage, int l0) {
+    if (live)
+      for (int l = l0; l < min(L, l0 + lc); ++l)
+#pragma unroll
+        for (int v = 0; v < VPT; ++v) {
+          const int vi = u + v * tpt;
+          if (vi < nvec)
+#pragma unroll
+            for (int q = 0; q < VB; ++q)
+              cp_async16(hslot(stage, l - l0, v) + q,
+                         reinterpret_cast<const uint4*>(hp + (int64_t)l * p.D + vi * 8) + q);
+        }
+    cp_async_commit();
+  };
   pdl_wait();
+  stage_chunk(0, 0);
+  stage_chunk(1, lc);
   const T* br = reinterpret_cast<const T*>(p.br[X]);
   for (int i = tid; i < tb * nj * L; i += blockDim.x) {
     const int tt = i / (nj * L), rem = i % (nj * L);
@@ -423,7 +465,6 @@ __global__ void __launch_bounds__(kMixThreads) mix_tokens_kernel(const MixParams
   }
   __syncthreads();
 
-  const T* hp = reinterpret_cast<const T*>(p.h) + (int64_t)b * L * p.D;
   const T* g = reinterpret_cast<const T*>(p.pre_g[X]);
   float gv[VPT][8];
   float acc[kMixCG][VPT][8];
@@ -436,10 +477,12 @@ __global__ void __launch_bounds__(kMixThreads) mix_tokens_kernel(const MixParams
 #pragma unroll
       for (int i = 0; i < 8; ++i) acc[jj][v][i] = 0.f;
   }
-  if (live) {
+  {
     const float* al = alpha + t * kMixCG * L;
-#pragma unroll 2
-    for (int l = 0; l < L; ++l) {
+    for (int l0 = 0, c = 0; l0 < L; l0 += lc, ++c) {
+      cp_async_wait<1>();  // this thread's copies of chunk c have landed
+      for (int l = l0; l < min(L, l0 + lc); ++l) {
+      if (!live) break;
       const float r = rl[t * L + l];
       float a[kMixCG];
 #pragma unroll
@@ -449,7 +492,7 @@ __global__ void __launch_bounds__(kMixThreads) mix_tokens_kernel(const MixParams
         const int vi = u + v * tpt;
         if (vi < nvec) {
           float hv[8];
-          load8f<T>(hp + (int64_t)l * p.D + vi * 8, hv);
+          load8f<T>(reinterpret_cast<const T*>(hslot(c & 1, l - l0, v)), hv);
 #pragma unroll
           for (int i = 0; i < 8; ++i) {
             const float hh = hv[i] * r * gv[v][i];  // pre-mix RMSNorm with gain
@@ -458,7 +501,10 @@ __global__ void __launch_bounds__(kMixThreads) mix_tokens_kernel(const MixParams
           }
         }
       }
+      }
+      stage_chunk(c & 1, l0 + 2 * lc);  // refill the buffer just consumed
     }
+    cp_async_wait<0>();
   }
   // per-channel sums of squares over the token's warps
 #pragma unroll
@@ -601,11 +647,21 @@ cudaError_t launch_all(MixParams& p, cudaStream_t s) {
     const int per = two ? (nvec + 1) / 2 : nvec;
     const int tpt = (per + 31) / 32 * 32;
     const int tb = tpt >= kMixThreads ? 1 : kMixThreads / tpt;
+    const size_t per_layer = (size_t)2 * (two ? 2 : 1) * tb * tpt * 8 * sizeof(T);  // both stages
+    int lc = kMixLC;
+    while (lc > 1 && (size_t)lc * per_layer > kMixStageBudget) lc /= 2;
     const size_t smem = sizeof(float) * ((size_t)tb * kMixCG * p.L + (size_t)tb * p.L +
-                                         (size_t)(tb * tpt / 32) * kMixCG);
+                                         (size_t)(tb * tpt / 32) * kMixCG) +
+                        16 + (size_t)lc * per_layer;
     dim3 grid((p.B + tb - 1) / tb, 2, (p.k + kMixCG - 1) / kMixCG);
-    e = two ? launch_pdl(mix_tokens_kernel<T, 2>, grid, dim3(tb * tpt), smem, s, p, tpt, tb)
-            : launch_pdl(mix_tokens_kernel<T, 1>, grid, dim3(tb * tpt), smem, s, p, tpt, tb);
+    auto kern = two ? mix_tokens_kernel<T, 2> : mix_tokens_kernel<T, 1>;
+    static size_t smem_set[2] = {0, 0};  // largest dynamic smem opted into, per variant
+    if (smem > smem_set[two]) {
+      e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+      if (e != cudaSuccess) return e;
+      smem_set[two] = smem;
+    }
+    e = launch_pdl(kern, grid, dim3(tb * tpt), smem, s, p, tpt, tb, lc);
     if (e != cudaSuccess) return e;
   } else {
     const size_t smem = sizeof(float) * (kChanGroup * p.L + p.L);

@@ -55,3 +55,24 @@ def test_batched_pool_over_several_token_tiles(B, g):
         assert H.rel_err(gv, v) <= H.TOL[w.dtype], ("V", b, j, H.rel_err(gv, v))
     torch.cuda.synchronize()
     torch.cuda.empty_cache()
+
+
+@pytest.mark.parametrize("dtype,D,B,L,k", [("f32", 256, 96, 4, 2), ("f32", 3072, 70, 4, 2),
+                                           ("bf16", 4096, 64, 6, 3)])
+def test_batched_pool_dtypes_and_widths(dtype, D, B, L, k):
+    """The batched forms of the pool (64 tokens and up) in fp32 and bf16, at
+    widths where a thread owns one or two 8-element vectors of D."""
+    w = configs.Workload("pool", L=L, k=k, D=D, Hq=2, Hkv=2, d=64, B=B, ctx=40, page=16,
+                         dtype=dtype, chan_map="mod", permute_pages=True, gain_std=0.1)
+    prob, sess, dp = H.setup(w, fill_pools=False)
+    sess.kv_mix(dp.h, dp.page_table, dp.slot)
+    torch.cuda.synchronize()
+    assert sess.read_status() == 0
+    tokens = [0, 1, B // 2, B - 1]
+    want = H.oracle_mix_tokens(prob, tokens=tokens)
+    for (b, j), (kk, vv) in want.items():
+        gk, gv = H.gpu_written_kv(sess, prob, b, j)
+        assert H.rel_err(gk, kk) <= H.TOL[dtype], ("K", b, j, H.rel_err(gk, kk))
+        assert H.rel_err(gv, vv) <= H.TOL[dtype], ("V", b, j, H.rel_err(gv, vv))
+    torch.cuda.synchronize()
+    torch.cuda.empty_cache()

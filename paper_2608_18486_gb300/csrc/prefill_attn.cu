@@ -10,6 +10,10 @@
 // this architecture.  One CTA (10 warps, one per SM) owns two 128-row query
 // tiles of one query head and walks the 128-slot KV tiles of the sequence's
 // channel up to each tile's largest position:
+//    With grouped-query attention (an even number G of query heads per kv
+//    head) the two tiles are the same 128 rows of two query heads that share
+//    a kv head: equal causal ranges, and one K/V stream serves both.
+//    Otherwise they are two consecutive 128-row tiles of one head.
 //  * warp 8 (TMA): the two Q tiles once, then K and V of every KV tile
 //    through separate rings (128-byte swizzle, 64-column boxes; paged: one
 //    box per page, or per 128 slots of a longer page);
@@ -65,6 +69,7 @@ struct PrefillParams {
   void* out;                  // [B][Tq][Hq][d] bf16
   int32_t* status;
   int32_t B, Tq, Hq, G, Hkv, chan, num_pages, max_pages, P, log2P;
+  int32_t pair;               // 1: the two tiles are query heads 2y, 2y+1 over the same rows
   float qscale;               // log2(e) / sqrt(d)
 };
 
@@ -88,9 +93,18 @@ __global__ void __launch_bounds__(kPThreads, 1)
   __shared__ int wmax[kSoftWarps];
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int b = blockIdx.z, hq = blockIdx.y, hkv = hq / p.G;
-  const int nblk = (p.Tq + kQT * kPM - 1) / (kQT * kPM);
-  const int r0 = (nblk - 1 - (int)blockIdx.x) * kQT * kPM;  // later rows (more work) first
+  // query tile i: rows rb[i] .. rb[i] + 127 of query head hh[i]
+  const int b = blockIdx.z;
+  const int rows_cta = p.pair ? kPM : kQT * kPM;
+  const int nblk = (p.Tq + rows_cta - 1) / rows_cta;
+  const int r0 = (nblk - 1 - (int)blockIdx.x) * rows_cta;  // later rows (more work) first
+  int rb[kQT], hh[kQT];
+#pragma unroll
+  for (int i = 0; i < kQT; ++i) {
+    rb[i] = p.pair ? r0 : r0 + i * kPM;
+    hh[i] = p.pair ? kQT * (int)blockIdx.y + i : (int)blockIdx.y;
+  }
+  const int hkv = hh[0] / p.G;  // the same kv head for both tiles
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_dyn) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
   uint8_t* Qs = base;                         // [kQT] Q tiles
@@ -129,7 +143,8 @@ __global__ void __launch_bounds__(kPThreads, 1)
   // ---- positions of the softmax threads' rows; the largest of each tile
   const int max_slots = p.max_pages * p.P;
   int mypos = -1;  // -1: row absent or invalid, fully masked
-  const int r = r0 + tid;
+  const int my_tile = warp < kSoftWarps ? warp >> 2 : 0;
+  const int r = rb[my_tile] + (tid - my_tile * kPM);
   if (warp < kSoftWarps && r < p.Tq) {
     const int v = p.pos[(int64_t)b * p.Tq + r];
     if (v >= 0 && v < max_slots) mypos = v;
@@ -171,8 +186,8 @@ __global__ void __launch_bounds__(kPThreads, 1)
         for (int i = 0; i < kQT; ++i)
 #pragma unroll
           for (int cb = 0; cb < CB; ++cb)
-            tc::tma_load_2d(Qs + i * SH::Q_BYTES + cb * kBlock, &tmQ, hq * HD + cb * 64,
-                            b * p.Tq + r0 + i * kPM, &qbar);
+            tc::tma_load_2d(Qs + i * SH::Q_BYTES + cb * kBlock, &tmQ, hh[i] * HD + cb * 64,
+                            b * p.Tq + rb[i], &qbar);
       }
       const int boxes = p.P >= kPN ? 1 : kPN >> p.log2P;  // <= 16 for pages of >= 8 slots
       const int brows = p.P >= kPN ? kPN : p.P;
@@ -403,7 +418,7 @@ __global__ void __launch_bounds__(kPThreads, 1)
       report(p.status, WM_ERR_TIMEOUT);
     } else {
       __nv_bfloat16* dst =
-          reinterpret_cast<__nv_bfloat16*>(p.out) + (((int64_t)b * p.Tq + r) * p.Hq + hq) * HD;
+          reinterpret_cast<__nv_bfloat16*>(p.out) + (((int64_t)b * p.Tq + r) * p.Hq + hh[i]) * HD;
       const float inv = (n > 0 && l > 0.f) ? 1.f / l : 0.f;
       tc::fence_after_sync();
 #pragma unroll
@@ -455,7 +470,8 @@ cudaError_t launch_hd(const CUtensorMap& q, const CUtensorMap& k, const CUtensor
     attr_set = true;
   }
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3((p.Tq + kQT * kPM - 1) / (kQT * kPM), p.Hq, p.B);
+  const int rows_cta = p.pair ? kPM : kQT * kPM;
+  cfg.gridDim = dim3((p.Tq + rows_cta - 1) / rows_cta, p.pair ? p.Hq / kQT : p.Hq, p.B);
   cfg.blockDim = dim3(kPThreads);
   cfg.dynamicSmemBytes = PShape<HD>::SMEM;
   cfg.stream = s;
@@ -487,6 +503,7 @@ cudaError_t launch_prefill_attn(const PrefillLaunch& L, cudaStream_t s) {
   p.Tq = L.Tq;
   p.Hq = L.Hq;
   p.G = L.Hq / L.Hkv;
+  p.pair = (p.G % kQT == 0) ? 1 : 0;
   p.Hkv = L.Hkv;
   p.chan = L.chan;
   p.num_pages = L.num_pages;

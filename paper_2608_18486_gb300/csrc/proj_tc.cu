@@ -15,9 +15,10 @@
 // last head are computed and ignored).  The work is
 // weight-streaming bound; TMA brings 128x64 weight tiles and Nx64 token
 // tiles (128-byte swizzle) through a 4-stage mbarrier pipeline.  Warp 0 lane
-// 0 issues TMA, warp 1 lane 0 issues tcgen05.mma; all four warps drain TMEM
-// (each warp its 32-lane quadrant) into shared memory, then finish the
-// per-(token, head) epilogue with a warp per item.
+// 0 issues TMA, warp 1 lane 0 issues tcgen05.mma, warps 2-7 fetch what the
+// epilogue needs; all eight warps drain TMEM (warps w and w + 4 share the
+// 32-lane quadrant w % 4) into shared memory, then finish the per-(token,
+// head) epilogue, several items per warp at a time.
 #include <cudaTypedefs.h>
 #include <math.h>
 
@@ -31,7 +32,7 @@ namespace {
 constexpr int kTcM = 128;      // weight rows per tile (MMA M)
 constexpr int kTcBK = 64;      // K elements per stage (128 bytes of bf16)
 constexpr int kTcMaxStages = 12;
-constexpr int kTcThreads = 128;
+constexpr int kTcThreads = 256;
 constexpr int kTcMaxTokens = 256;
 
 enum { kEpiKV = 0, kEpiPartial = 1 };
@@ -123,10 +124,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   } else if (MODE == kEpiKV && warp >= 2) {
     // meanwhile warps 2-3 fetch what the epilogue needs: the RoPE table of the
     // tile's tokens and each token's destination slot and page
-    const int t2 = threadIdx.x - 64;
+    const int t2 = threadIdx.x - 64, n2 = kTcThreads - 64;
     if (p.rope_smem_off > 0)
-      for (int i = t2; i < nb * HD; i += 64) rope_s[i] = p.rope_cs[(int64_t)n0 * HD + i];
-    for (int n = t2; n < nb; n += 64) {
+      for (int i = t2; i < nb * HD; i += n2) rope_s[i] = p.rope_cs[(int64_t)n0 * HD + i];
+    for (int n = t2; n < nb; n += n2) {
       const int s = p.slot[n0 + n];
       int pg = -1;
       if (s >= 1 && s < p.max_pages * p.P)
@@ -153,16 +154,17 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     }
     tc::mma_commit(&done);  // always issued: fires when every MMA above is complete
   }
-  const bool ok = mbar_wait(&done, 0);
-  __syncwarp();
+  // warp-uniform: the TMEM loads below are warp-collective
+  const bool ok = __all_sync(0xFFFFFFFFu, mbar_wait(&done, 0));
   tc::fence_after_sync();
 
-  // TMEM -> shared tile T[token][row] (fp32); the stage buffers are free now
+  // TMEM -> shared tile T[token][row] (fp32); the stage buffers are free now.
+  // Warps w and w + 4 share lane quadrant w % 4 and split its columns.
   float* T = reinterpret_cast<float*>(base);
   if (ok) {
-    const uint32_t quad = (uint32_t)(warp * 32) << 16;
-    const int row = warp * 32 + lane;
-    for (int c0 = 0; c0 < p.BN; c0 += 16) {
+    const uint32_t quad = (uint32_t)((warp & 3) * 32) << 16;
+    const int row = (warp & 3) * 32 + lane;
+    for (int c0 = (warp >> 2) * 16; c0 < p.BN; c0 += 32) {
       uint32_t r[16];
       tc::tmem_ld16(tmem + quad + (uint32_t)c0, r);
       tc::tmem_ld_wait();

@@ -219,6 +219,7 @@ __global__ void __launch_bounds__(kThreads, attn_ctas_per_sm(SB, G)) decode_attn
   constexpr uint32_t KV_BYTES = STAGE_ELEMS * sizeof(T);
   constexpr uint32_t Q_BYTES = G * HD * sizeof(T);
   constexpr int REC = attn_part_rec(G, HD);                        // floats per partial record
+  constexpr int FLAG = G * HD + 2 * G;                             // the record's "published" word
   constexpr int RING_RECS = (int)(kWStages * 2 * KV_BYTES / (REC * sizeof(float)));
   static_assert(RING_RECS >= 1 && (REC * sizeof(float)) % 16 == 0, "partial records");
   // Partial merges take pieces in batches of MB (every load of a batch issued
@@ -531,44 +532,74 @@ __global__ void __launch_bounds__(kThreads, attn_ctas_per_sm(SB, G)) decode_attn
       if (g_first == g_last) {
         if (lane_slot == 0) write_rows<T, HD, G, SB>(outp + rowbase * HD, lane_part, st);
       } else {
-        // partial of this piece: its chunk's first piece -> side 0, last piece -> side 1
-        for (int side = 0; side < 2; ++side) {
-          if ((side == 0 && !piece_first) || (side == 1 && !chunk_end)) continue;
-          float* po = p.part + ((int64_t)side * p.max_chunks + c_chunk) * REC;
-          float* pm = po + G * HD;
-          if (lane_slot == 0) {
+        // Records of the unit's pieces: side 1 of chunk g_first, then side 0 of
+        // g_first + 1 .. g_last (consecutive).  Each warp takes its ticket
+        // first; the one that completes the unit merges, the others publish
+        // their record and then set its flag (the word after the (m, l)
+        // pairs) to this call's epoch, so the merging warp never publishes its
+        // own piece.  The merger clears the flags it consumed (a CUDA graph
+        // replays a call with the same epoch).
+        const int np = (int)(g_last - g_first + 1);
+        const int j_own = (int)(c_chunk - g_first);  // this piece's record in the merge
+        const float* rec1 = p.part + (int64_t)(p.max_chunks + g_first) * REC;
+        const float* rec0 = p.part + (int64_t)(g_first + 1) * REC;
+        auto rec_of = [&](int j) -> const float* { return j == 0 ? rec1 : rec0 + (int64_t)(j - 1) * REC; };
+        auto flag_of = [&](const float* r) -> volatile int* {
+          return reinterpret_cast<volatile int*>(const_cast<float*>(r) + FLAG);
+        };
+        // this piece's partial as records: its chunk's first piece -> side 0,
+        // last piece -> side 1
+        auto write_records = [&](bool raise_flags) {
+          for (int side = 0; side < 2; ++side) {
+            if ((side == 0 && !piece_first) || (side == 1 && !chunk_end)) continue;
+            float* po = p.part + ((int64_t)side * p.max_chunks + c_chunk) * REC;
+            float* pm = po + G * HD;
+            if (lane_slot == 0) {
 #pragma unroll
-            for (int g = 0; g < G; ++g)
+              for (int g = 0; g < G; ++g)
 #pragma unroll
-              for (int v = 0; v < SH::NVL; ++v)
+                for (int v = 0; v < SH::NVL; ++v)
 #pragma unroll
-                for (int i = 0; i < VEC / 2; ++i)
-                  reinterpret_cast<float2*>(po + g * HD + (v * LPS + lane_part) * VEC)[i] =
-                      st.acc[g][v * VEC / 2 + i];
-          }
-          if (lane == 0) {
+                  for (int i = 0; i < VEC / 2; ++i)
+                    reinterpret_cast<float2*>(po + g * HD + (v * LPS + lane_part) * VEC)[i] =
+                        st.acc[g][v * VEC / 2 + i];
+            }
+            if (lane == 0) {
 #pragma unroll
-            for (int g = 0; g < G; ++g) {
-              pm[2 * g] = st.m[g];
-              pm[2 * g + 1] = st.l[g];
+              for (int g = 0; g < G; ++g) {
+                pm[2 * g] = st.m[g];
+                pm[2 * g + 1] = st.l[g];
+              }
             }
           }
-        }
-        __threadfence();
-        __syncwarp();
-        int last = 0;
-        if (lane == 0) {
-          const int t = atomicAdd(&p.counters[cc.b * Hkv + cc.h], 1);
-          last = (t == (int)(g_last - g_first));
-        }
-        last = __shfl_sync(FULLMASK, last, 0);
-        if (last) {
           __threadfence();
-          // merge the pieces of chunks g_first .. g_last: side 1 of the first
-          // chunk, then side 0 of the others (consecutive records)
-          const int np = (int)(g_last - g_first + 1);
-          const float* rec1 = p.part + (int64_t)(p.max_chunks + g_first) * REC;
-          const float* rec0 = p.part + (int64_t)(g_first + 1) * REC;
+          __syncwarp();
+          if (raise_flags && lane == 0) {
+            if (piece_first) *flag_of(p.part + (int64_t)c_chunk * REC) = p.epoch;
+            if (chunk_end) *flag_of(p.part + ((int64_t)p.max_chunks + c_chunk) * REC) = p.epoch;
+          }
+        };
+        int last = 0;
+        if (lane == 0) last = atomicAdd(&p.counters[cc.b * Hkv + cc.h], 1) == np - 1;
+        last = __shfl_sync(FULLMASK, last, 0);
+        if (!last) {
+          write_records(true);
+        } else {
+          // every other piece has its ticket and only has its stores left:
+          // wait (bounded) for their flags
+          bool ready = false;
+          const uint64_t t0 = globaltimer_ns();
+          for (uint32_t it = 0;; ++it) {
+            bool mine = true;
+            for (int j = lane; j < np; j += 32)
+              if (j != j_own) mine = mine && (*flag_of(rec_of(j)) == p.epoch);
+            ready = __all_sync(FULLMASK, mine);
+            if (ready || ((it & 63u) == 63u && globaltimer_ns() - t0 > kWaitLimitNs)) break;
+          }
+          if (!ready) {
+            if (lane == 0) report(p.status, WM_ERR_TIMEOUT);
+          } else {
+          __threadfence();
           if (p_done && seq + 1 == pseq) {
             // no stage in flight: the ring takes ROUND records per round
             float* rs = reinterpret_cast<float*>(myring);
@@ -605,6 +636,28 @@ __global__ void __launch_bounds__(kThreads, attn_ctas_per_sm(SB, G)) decode_attn
                 }
                 landed = false;
                 break;
+              }
+              if (j_own >= r0 && j_own < r0 + n) {
+                // this warp's own piece was never published: take it from registers
+                float* ro = rs + (j_own - r0) * REC;
+                if (lane_slot == 0) {
+#pragma unroll
+                  for (int g = 0; g < G; ++g)
+#pragma unroll
+                    for (int v = 0; v < SH::NVL; ++v)
+#pragma unroll
+                      for (int i = 0; i < VEC / 2; ++i)
+                        reinterpret_cast<float2*>(ro + g * HD + (v * LPS + lane_part) * VEC)[i] =
+                            st.acc[g][v * VEC / 2 + i];
+                }
+                if (lane == 0) {
+#pragma unroll
+                  for (int g = 0; g < G; ++g) {
+                    ro[G * HD + 2 * g] = st.m[g];
+                    ro[G * HD + 2 * g + 1] = st.l[g];
+                  }
+                }
+                __syncwarp();
               }
 #pragma unroll
               for (int g = 0; g < G; ++g) {
@@ -649,6 +702,8 @@ __global__ void __launch_bounds__(kThreads, attn_ctas_per_sm(SB, G)) decode_attn
             }
           } else {
             // stages in flight: the same batches, straight from global memory
+            // (this warp's own records first, for its other lanes to read)
+            write_records(false);
             for (int g = 0; g < G; ++g) {
               float M = -INFINITY, Ls = 0.f;
               float o[HD / 32];
@@ -691,7 +746,11 @@ __global__ void __launch_bounds__(kThreads, attn_ctas_per_sm(SB, G)) decode_attn
                 outp[(rowbase + g) * HD + lane + 32 * i] = Elem<T>::from_f(o[i] * inv);
             }
           }
+          // ready for the next launch: flags down, ticket counter zero
+          for (int j = lane; j < np; j += 32)
+            if (j != j_own) *flag_of(rec_of(j)) = 0;
           if (lane == 0) p.counters[cc.b * Hkv + cc.h] = 0;
+          }
         }
       }
       piece_first = false;

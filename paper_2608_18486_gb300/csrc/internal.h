@@ -18,7 +18,8 @@ struct AttnParams {
   const int32_t* seq_lens;
   float* part;            // [2][max_chunks] records of attn_part_rec(G, d) floats: the
                           // first / last piece partial of each chunk ([G][d] unnormalised
-                          // outputs, then (max, sum) per query head in log2 units)
+                          // outputs, (max, sum) per query head in log2 units, then a
+                          // published flag, zero between launches)
   int32_t* counters;      // [B*Hkv] arrival tickets + 1 chunk counter, zero between launches
   int32_t* status;
   int64_t page_stride;    // elements between consecutive physical pages
@@ -26,6 +27,9 @@ struct AttnParams {
   int32_t chunk_stages;   // stages per work chunk (0: one chunk per warp)
   int32_t max_chunks;     // partial slots per side
   int32_t inputs_ready;   // the previous grid wrote no cache, table, length or workspace
+  int32_t epoch;          // nonzero tag of this call: a record is published when its
+                          // flag holds this value (a stale word from another call or
+                          // layout never matches)
   float qscale;           // log2(e) / sqrt(d)
 };
 
@@ -33,9 +37,10 @@ struct AttnParams {
 // and one query head per kv head, else 2 (GQA keeps G query rows per lane).
 constexpr int attn_ctas_per_sm(int stage_bytes, int G) { return stage_bytes == 4096 && G == 1 ? 4 : 2; }
 
-// Floats per partial record: G*d outputs, then (max, sum) per head, padded to
-// 16 bytes so that consecutive records can be moved with one bulk copy.
-constexpr int attn_part_rec(int G, int d) { return G * d + (2 * G > 4 ? 2 * G : 4); }
+// Floats per partial record: G*d outputs, (max, sum) per head, a "published"
+// flag word, padded to 16 bytes so that consecutive records can be moved with
+// one bulk copy.
+constexpr int attn_part_rec(int G, int d) { return G * d + (2 * G + 1 + 3) / 4 * 4; }
 
 int attn_stage_slots(int stage_bytes, int dtype, int d);
 int attn_warps_per_cta();

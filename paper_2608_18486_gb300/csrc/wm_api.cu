@@ -3,6 +3,7 @@
 #include <math.h>
 #include <string.h>
 
+#include <atomic>
 #include <mutex>
 
 #include "common.cuh"
@@ -90,6 +91,17 @@ AttnPlan attn_plan(const wm_config& c, int32_t B, int32_t max_pages) {
   off += align256(sizeof(int32_t) * ((size_t)B * c.Hkv + 1));
   pl.total = off;
   return pl;
+}
+
+// Tag of one attention call (never 0): a partial record counts as published
+// only when its flag holds the tag of the call reading it.
+int32_t next_attn_epoch() {
+  static std::atomic<uint32_t> counter{0};
+  uint32_t e;
+  do {
+    e = counter.fetch_add(1, std::memory_order_relaxed) + 1;
+  } while ((e & 0x7FFFFFFFu) == 0);
+  return (int32_t)(e & 0x7FFFFFFFu);
 }
 
 wm_status check_cache(const wm_config& c, const wm_cache* cache) {
@@ -216,6 +228,7 @@ wm_status wm_decode_attn_flags(const wm_config* c, const wm_cache* cache, int32_
   p.chunk_stages = pl.chunk_stages;
   p.max_chunks = pl.max_chunks;
   p.inputs_ready = (flags & WM_ATTN_INPUTS_READY) ? 1 : 0;
+  p.epoch = next_attn_epoch();
   p.qscale = (float)(1.4426950408889634 / sqrt((double)c->d));
   cudaError_t e = wm::launch_decode_attn(p, pl.stage_bytes, c->dtype, c->d, c->Hq / c->Hkv,
                                          pl.grid, (cudaStream_t)stream);

@@ -22,11 +22,14 @@
 //    shuffles at the end of a piece.
 //  * Merge.  A piece of a unit that lies inside one chunk is written straight
 //    to the output.  Only units that cross a chunk boundary leave partials
-//    (at most two per chunk: its first and its last piece); the last warp to
-//    finish such a unit (atomic ticket, no waiting) merges them.  When that
-//    warp has no stage left in flight, its idle ring receives the unit's
-//    partial records with bulk copies (one round trip for up to a ring's
-//    worth), and the merge reads them from shared memory.
+//    (at most two per chunk: its first and its last piece).  A warp takes
+//    its ticket on the unit first: the warp that completes the unit merges,
+//    every other one publishes its partial and then flags it, so the merger
+//    never publishes its own piece and waits (bounded) only for flags that
+//    are in flight.  When the merger has no stage left in flight, its idle
+//    ring receives the unit's partial records with bulk copies (one round
+//    trip for up to a ring's worth), and the merge reads them from shared
+//    memory.
 #include <math.h>
 
 #include "common.cuh"
@@ -599,157 +602,157 @@ __global__ void __launch_bounds__(kThreads, attn_ctas_per_sm(SB, G)) decode_attn
           if (!ready) {
             if (lane == 0) report(p.status, WM_ERR_TIMEOUT);
           } else {
-          __threadfence();
-          if (p_done && seq + 1 == pseq) {
-            // no stage in flight: the ring takes ROUND records per round
-            float* rs = reinterpret_cast<float*>(myring);
-            float M[G], Ls[G], o[G][HD / 32];
-#pragma unroll
-            for (int g = 0; g < G; ++g) {
-              M[g] = -INFINITY;
-              Ls[g] = 0.f;
-#pragma unroll
-              for (int i = 0; i < HD / 32; ++i) o[g][i] = 0.f;
-            }
-            fence_proxy_async_global();
-            fence_proxy_async_shared();
-            bool landed = true;
-            for (int r0 = 0; r0 < np; r0 += ROUND) {
-              const int n = min(ROUND, np - r0);
-              constexpr uint32_t RB = REC * sizeof(float);
-              if (lane == 0) {
-                mbar_arrive_expect_tx(&qbars[warp], (uint32_t)n * RB);
-                if (r0 == 0) {
-                  bulk_g2s(rs, rec1, RB, &qbars[warp], policy);
-                  if (n > 1) bulk_g2s(rs + REC, rec0, (uint32_t)(n - 1) * RB, &qbars[warp], policy);
-                } else {
-                  bulk_g2s(rs, rec0 + (int64_t)(r0 - 1) * REC, (uint32_t)n * RB, &qbars[warp], policy);
-                }
-              }
-              // qbars completed phase 0 with the first query; round r is phase r + 1
-              const uint32_t parity = (uint32_t)(r0 / ROUND + 1) & 1u;
-              landed = mbar_wait(&qbars[warp], parity);
-              if (__any_sync(FULLMASK, !landed)) {
-                if (lane == 0) {
-                  report(p.status, WM_ERR_TIMEOUT);
-                  mbar_wait(&qbars[warp], parity);
-                }
-                landed = false;
-                break;
-              }
-              if (j_own >= r0 && j_own < r0 + n) {
-                // this warp's own piece was never published: take it from registers
-                float* ro = rs + (j_own - r0) * REC;
-                if (lane_slot == 0) {
-#pragma unroll
-                  for (int g = 0; g < G; ++g)
-#pragma unroll
-                    for (int v = 0; v < SH::NVL; ++v)
-#pragma unroll
-                      for (int i = 0; i < VEC / 2; ++i)
-                        reinterpret_cast<float2*>(ro + g * HD + (v * LPS + lane_part) * VEC)[i] =
-                            st.acc[g][v * VEC / 2 + i];
-                }
-                if (lane == 0) {
-#pragma unroll
-                  for (int g = 0; g < G; ++g) {
-                    ro[G * HD + 2 * g] = st.m[g];
-                    ro[G * HD + 2 * g + 1] = st.l[g];
-                  }
-                }
-                __syncwarp();
-              }
+            __threadfence();
+            if (p_done && seq + 1 == pseq) {
+              // no stage in flight: the ring takes ROUND records per round
+              float* rs = reinterpret_cast<float*>(myring);
+              float M[G], Ls[G], o[G][HD / 32];
 #pragma unroll
               for (int g = 0; g < G; ++g) {
-                for (int b0 = 0; b0 < n; b0 += MB) {
-                  float mq[MB], lq[MB];
+                M[g] = -INFINITY;
+                Ls[g] = 0.f;
+#pragma unroll
+                for (int i = 0; i < HD / 32; ++i) o[g][i] = 0.f;
+              }
+              fence_proxy_async_global();
+              fence_proxy_async_shared();
+              bool landed = true;
+              for (int r0 = 0; r0 < np; r0 += ROUND) {
+                const int n = min(ROUND, np - r0);
+                constexpr uint32_t RB = REC * sizeof(float);
+                if (lane == 0) {
+                  mbar_arrive_expect_tx(&qbars[warp], (uint32_t)n * RB);
+                  if (r0 == 0) {
+                    bulk_g2s(rs, rec1, RB, &qbars[warp], policy);
+                    if (n > 1) bulk_g2s(rs + REC, rec0, (uint32_t)(n - 1) * RB, &qbars[warp], policy);
+                  } else {
+                    bulk_g2s(rs, rec0 + (int64_t)(r0 - 1) * REC, (uint32_t)n * RB, &qbars[warp], policy);
+                  }
+                }
+                // qbars completed phase 0 with the first query; round r is phase r + 1
+                const uint32_t parity = (uint32_t)(r0 / ROUND + 1) & 1u;
+                landed = mbar_wait(&qbars[warp], parity);
+                if (__any_sync(FULLMASK, !landed)) {
+                  if (lane == 0) {
+                    report(p.status, WM_ERR_TIMEOUT);
+                    mbar_wait(&qbars[warp], parity);
+                  }
+                  landed = false;
+                  break;
+                }
+                if (j_own >= r0 && j_own < r0 + n) {
+                  // this warp's own piece was never published: take it from registers
+                  float* ro = rs + (j_own - r0) * REC;
+                  if (lane_slot == 0) {
+#pragma unroll
+                    for (int g = 0; g < G; ++g)
+#pragma unroll
+                      for (int v = 0; v < SH::NVL; ++v)
+#pragma unroll
+                        for (int i = 0; i < VEC / 2; ++i)
+                          reinterpret_cast<float2*>(ro + g * HD + (v * LPS + lane_part) * VEC)[i] =
+                              st.acc[g][v * VEC / 2 + i];
+                  }
+                  if (lane == 0) {
+#pragma unroll
+                    for (int g = 0; g < G; ++g) {
+                      ro[G * HD + 2 * g] = st.m[g];
+                      ro[G * HD + 2 * g + 1] = st.l[g];
+                    }
+                  }
+                  __syncwarp();
+                }
+#pragma unroll
+                for (int g = 0; g < G; ++g) {
+                  for (int b0 = 0; b0 < n; b0 += MB) {
+                    float mq[MB], lq[MB];
+#pragma unroll
+                    for (int jb = 0; jb < MB; ++jb) {
+                      const bool in = b0 + jb < n;
+                      mq[jb] = in ? rs[(b0 + jb) * REC + G * HD + 2 * g] : -INFINITY;
+                      lq[jb] = in ? rs[(b0 + jb) * REC + G * HD + 2 * g + 1] : 0.f;
+                    }
+                    float Mn = M[g];
+#pragma unroll
+                    for (int jb = 0; jb < MB; ++jb) Mn = fmaxf(Mn, mq[jb]);
+                    if (Mn == -INFINITY) continue;
+                    const float rescale = exp2f(M[g] - Mn);  // 0 on the first batch
+                    Ls[g] *= rescale;
+#pragma unroll
+                    for (int i = 0; i < HD / 32; ++i) o[g][i] *= rescale;
+#pragma unroll
+                    for (int jb = 0; jb < MB; ++jb) {
+                      if (mq[jb] == -INFINITY) continue;
+                      const float w = exp2f(mq[jb] - Mn);
+                      Ls[g] = fmaf(w, lq[jb], Ls[g]);
+                      const float* rj = rs + (b0 + jb) * REC + g * HD + lane;
+#pragma unroll
+                      for (int i = 0; i < HD / 32; ++i) o[g][i] = fmaf(w, rj[32 * i], o[g][i]);
+                    }
+                    M[g] = Mn;
+                  }
+                }
+                __syncwarp();  // every lane is done with the ring before the next round
+              }
+              if (landed) {
+#pragma unroll
+                for (int g = 0; g < G; ++g) {
+                  const float inv = Ls[g] > 0.f ? 1.f / Ls[g] : 0.f;
+#pragma unroll
+                  for (int i = 0; i < HD / 32; ++i)
+                    outp[(rowbase + g) * HD + lane + 32 * i] = Elem<T>::from_f(o[g][i] * inv);
+                }
+              }
+            } else {
+              // stages in flight: the same batches, straight from global memory
+              // (this warp's own records first, for its other lanes to read)
+              write_records(false);
+              for (int g = 0; g < G; ++g) {
+                float M = -INFINITY, Ls = 0.f;
+                float o[HD / 32];
+#pragma unroll
+                for (int i = 0; i < HD / 32; ++i) o[i] = 0.f;
+                for (int r0 = 0; r0 < np; r0 += MB) {
+                  float mq[MB], lq[MB], ov[MB][HD / 32];
 #pragma unroll
                   for (int jb = 0; jb < MB; ++jb) {
-                    const bool in = b0 + jb < n;
-                    mq[jb] = in ? rs[(b0 + jb) * REC + G * HD + 2 * g] : -INFINITY;
-                    lq[jb] = in ? rs[(b0 + jb) * REC + G * HD + 2 * g + 1] : 0.f;
+                    const int j = r0 + jb;
+                    const bool in = j < np;
+                    const float* rj = j == 0 ? rec1 : rec0 + (int64_t)(j - 1) * REC;
+                    mq[jb] = in ? __ldcg(rj + G * HD + 2 * g) : -INFINITY;
+                    lq[jb] = in ? __ldcg(rj + G * HD + 2 * g + 1) : 0.f;
+#pragma unroll
+                    for (int i = 0; i < HD / 32; ++i)
+                      ov[jb][i] = in ? __ldcg(rj + g * HD + lane + 32 * i) : 0.f;
                   }
-                  float Mn = M[g];
+                  float Mn = M;
 #pragma unroll
                   for (int jb = 0; jb < MB; ++jb) Mn = fmaxf(Mn, mq[jb]);
                   if (Mn == -INFINITY) continue;
-                  const float rescale = exp2f(M[g] - Mn);  // 0 on the first batch
-                  Ls[g] *= rescale;
+                  const float rescale = exp2f(M - Mn);  // 0 on the first batch
+                  Ls *= rescale;
 #pragma unroll
-                  for (int i = 0; i < HD / 32; ++i) o[g][i] *= rescale;
+                  for (int i = 0; i < HD / 32; ++i) o[i] *= rescale;
 #pragma unroll
                   for (int jb = 0; jb < MB; ++jb) {
                     if (mq[jb] == -INFINITY) continue;
                     const float w = exp2f(mq[jb] - Mn);
-                    Ls[g] = fmaf(w, lq[jb], Ls[g]);
-                    const float* rj = rs + (b0 + jb) * REC + g * HD + lane;
+                    Ls = fmaf(w, lq[jb], Ls);
 #pragma unroll
-                    for (int i = 0; i < HD / 32; ++i) o[g][i] = fmaf(w, rj[32 * i], o[g][i]);
+                    for (int i = 0; i < HD / 32; ++i) o[i] = fmaf(w, ov[jb][i], o[i]);
                   }
-                  M[g] = Mn;
+                  M = Mn;
                 }
-              }
-              __syncwarp();  // every lane is done with the ring before the next round
-            }
-            if (landed) {
-#pragma unroll
-              for (int g = 0; g < G; ++g) {
-                const float inv = Ls[g] > 0.f ? 1.f / Ls[g] : 0.f;
+                const float inv = Ls > 0.f ? 1.f / Ls : 0.f;
 #pragma unroll
                 for (int i = 0; i < HD / 32; ++i)
-                  outp[(rowbase + g) * HD + lane + 32 * i] = Elem<T>::from_f(o[g][i] * inv);
+                  outp[(rowbase + g) * HD + lane + 32 * i] = Elem<T>::from_f(o[i] * inv);
               }
             }
-          } else {
-            // stages in flight: the same batches, straight from global memory
-            // (this warp's own records first, for its other lanes to read)
-            write_records(false);
-            for (int g = 0; g < G; ++g) {
-              float M = -INFINITY, Ls = 0.f;
-              float o[HD / 32];
-#pragma unroll
-              for (int i = 0; i < HD / 32; ++i) o[i] = 0.f;
-              for (int r0 = 0; r0 < np; r0 += MB) {
-                float mq[MB], lq[MB], ov[MB][HD / 32];
-#pragma unroll
-                for (int jb = 0; jb < MB; ++jb) {
-                  const int j = r0 + jb;
-                  const bool in = j < np;
-                  const float* rj = j == 0 ? rec1 : rec0 + (int64_t)(j - 1) * REC;
-                  mq[jb] = in ? __ldcg(rj + G * HD + 2 * g) : -INFINITY;
-                  lq[jb] = in ? __ldcg(rj + G * HD + 2 * g + 1) : 0.f;
-#pragma unroll
-                  for (int i = 0; i < HD / 32; ++i)
-                    ov[jb][i] = in ? __ldcg(rj + g * HD + lane + 32 * i) : 0.f;
-                }
-                float Mn = M;
-#pragma unroll
-                for (int jb = 0; jb < MB; ++jb) Mn = fmaxf(Mn, mq[jb]);
-                if (Mn == -INFINITY) continue;
-                const float rescale = exp2f(M - Mn);  // 0 on the first batch
-                Ls *= rescale;
-#pragma unroll
-                for (int i = 0; i < HD / 32; ++i) o[i] *= rescale;
-#pragma unroll
-                for (int jb = 0; jb < MB; ++jb) {
-                  if (mq[jb] == -INFINITY) continue;
-                  const float w = exp2f(mq[jb] - Mn);
-                  Ls = fmaf(w, lq[jb], Ls);
-#pragma unroll
-                  for (int i = 0; i < HD / 32; ++i) o[i] = fmaf(w, ov[jb][i], o[i]);
-                }
-                M = Mn;
-              }
-              const float inv = Ls > 0.f ? 1.f / Ls : 0.f;
-#pragma unroll
-              for (int i = 0; i < HD / 32; ++i)
-                outp[(rowbase + g) * HD + lane + 32 * i] = Elem<T>::from_f(o[i] * inv);
-            }
-          }
-          // ready for the next launch: flags down, ticket counter zero
-          for (int j = lane; j < np; j += 32)
-            if (j != j_own) *flag_of(rec_of(j)) = 0;
-          if (lane == 0) p.counters[cc.b * Hkv + cc.h] = 0;
+            // ready for the next launch: flags down, ticket counter zero
+            for (int j = lane; j < np; j += 32)
+              if (j != j_own) *flag_of(rec_of(j)) = 0;
+            if (lane == 0) p.counters[cc.b * Hkv + cc.h] = 0;
           }
         }
       }

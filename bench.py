@@ -197,6 +197,54 @@ def oracle_step_estimate(prob, budget_s: float = 4.0, nthreads: int | None = Non
     return attn_step + mix_step, cores, sample
 
 
+def oracle_prefill_estimate(prob, T: int, g: int, budget_s: float = 4.0):
+    """Time the fp64 oracle on a bounded sample of query rows of a prefill
+    pass and extrapolate by work (a row at position i reads i + 1 slots) to
+    every row, head and layer.  Returns (seconds per pass, cores, sample)."""
+    import numpy as np
+    from tests import _harness as H
+    from wm_synth import gen
+    from wm_synth.inputs import STREAM_Q_PREFILL
+    w = prob.w
+    rng = np.random.default_rng(0)
+    t_used, work, rows = 0.0, 0, 0
+    while t_used < budget_s:
+        b, pos, hq = int(rng.integers(w.B)), int(rng.integers(T)), int(rng.integers(w.Hq))
+        qv = gen.values(w.dtype, 0, STREAM_Q_PREFILL, rows * w.d, w.d, w.q_scale)
+        t = time.perf_counter()
+        H.oracle_prefill_unit(prob, 0, b, pos, (hq, qv))
+        t_used += time.perf_counter() - t
+        work += pos + 1
+        rows += 1
+    total = w.L * w.B * w.Hq * T * (T + 1) / 2.0
+    sample = (f"{rows} query rows at random positions (one head, layer 0; {work} slot reads), "
+              f"extrapolated by slots read to {w.L} layers x {w.B} sequences x {w.Hq} heads "
+              f"x {T} positions")
+    return t_used * total / max(work, 1), 1, sample
+
+
+def oracle_pool_estimate(prob, budget_s: float = 4.0, nthreads: int | None = None):
+    """Time the fp64 oracle's pool on whole tokens until the budget is spent
+    and extrapolate to B tokens.  Returns (seconds per pool, cores, sample)."""
+    import numpy as np
+    from oracle import oracle as O
+    w = prob.w
+    cores = nthreads or len(os.sched_getaffinity(0))
+    args = [prob.host(n) for n in ("pre_g", "Wr", "br", "ch_g", "Wkv", "qk_g")]
+    hall = prob.host("h")
+    t_mix, tok = 0.0, 0
+    while tok < w.B and t_mix < budget_s:
+        n = min(cores, w.B - tok)
+        h = hall[tok:tok + n]
+        pos = (prob.seq_lens[tok:tok + n] - 1).astype(np.float64)
+        t = time.perf_counter()
+        O.kv_mix(h, pos, *args, L=w.L, k=w.k, D=w.D, Hkv=w.Hkv, d=w.d, p=w.p, eps=w.eps_rms,
+                 eps_qk=w.eps_qk, theta=w.rope_theta, nthreads=cores)
+        t_mix += time.perf_counter() - t
+        tok += n
+    return t_mix * w.B / max(tok, 1), cores, f"pool for {tok} of {w.B} tokens, extrapolated by tokens"
+
+
 # ---------------------------------------------------------------- arms
 def run_reference(args, w):
     rank, world, _ = dist_env()
@@ -619,6 +667,9 @@ def run_prefill(args, w):
                          "frac": tflops / peak, "peak_kind": "measured sustained bf16",
                          "flops_per_step": flops},
             "clocks": clocks, "gpu_launches": K * w.L * g}
+    t_cpu, cores, sample = oracle_prefill_estimate(prob, T, g, budget_s=args.ref_budget)
+    line["cpu_baseline"] = {"value": w.B * T / t_cpu, "unit": "tokens/s", "cores": cores,
+                            "kind": "oracle", "sample": sample}
     print(json.dumps(line), flush=True)
 
 
@@ -689,7 +740,10 @@ def run_pool(args, w):
             "roofline": {"bound": "tensor", "achieved": tflops, "peak": peak, "unit": "TFLOP/s",
                          "frac": tflops / peak, "peak_kind": "measured sustained bf16",
                          "flops_per_step": flops, "bytes_per_step": wcfg.mix_bytes(w)},
-            "clocks": clocks}
+            "clocks": clocks, "gpu_launches": K * 4}
+    t_cpu, cores, sample = oracle_pool_estimate(prob, budget_s=args.ref_budget)
+    line["cpu_baseline"] = {"value": w.B / t_cpu, "unit": "tokens/s", "cores": cores,
+                            "kind": "oracle", "sample": sample}
     print(json.dumps(line), flush=True)
 
 

@@ -76,6 +76,28 @@ def oracle_attn_unit(prob, layer, b, hq) -> np.ndarray:
     return O.decode_attn(q, kp, vp, pt, [S], chan=0, Hq=1, Hkv=1, d=w.d, P=w.page)[0, 0]
 
 
+def oracle_prefill_unit(prob, layer, b, pos, q_row) -> np.ndarray:
+    """Causal prefill attention of one query row (token position ``pos`` of
+    sequence b, query head given by ``q_row``'s head index), from only the
+    pages it reads.  ``q_row`` is (hq, d storage-dtype values)."""
+    w = prob.w
+    hq, qv = q_row
+    hkv = hq // (w.Hq // w.Hkv)
+    chan = prob.chan[layer]
+    npg = pos // w.page + 1
+    pages = prob.page_table[b, :npg].astype(np.int64)
+    s = np.arange(w.page, dtype=np.int64)
+    e = np.arange(w.d, dtype=np.int64)
+    base = ((chan * prob.num_pages + pages) * w.Hkv + hkv) * w.page
+    idx = ((base[:, None] + s[None, :]) * w.d)[:, :, None] + e[None, None, :]
+    kp = prob.at("k_pool", idx.reshape(-1)).reshape(1, npg, 1, w.page, w.d)
+    vp = prob.at("v_pool", idx.reshape(-1)).reshape(1, npg, 1, w.page, w.d)
+    pt = np.arange(npg, dtype=np.int32).reshape(1, npg)
+    q = np.ascontiguousarray(qv).reshape(1, 1, 1, w.d)
+    return O.prefill_attn(q, kp, vp, pt, np.array([[pos]], np.int32), chan=0, Hq=1, Hkv=1,
+                          d=w.d, P=w.page)[0, 0, 0]
+
+
 def oracle_mix_tokens(prob, tokens=None, chans=None):
     """K~ and V of the chosen tokens and channels: dict[(b, j)] -> (K[Hkv][d], V[Hkv][d])."""
     w = prob.w

@@ -246,3 +246,20 @@ def test_inputs_ready_chain_matches_default_launches(name, overrides):
     if name == "no_compression":
         assert H.rel_err(H.to_f64(outs[3]), H.oracle_attn_full(prob, 3)) <= H.TOL[w.dtype]
     _free()
+
+
+def test_workspace_reused_across_batch_sizes():
+    """One workspace serves calls whose plans lay partial records out
+    differently (a smaller batch splits into fewer chunks): words left by
+    another call never pass for published records."""
+    w = configs.get("no_compression").with_(L=2, k=2)
+    prob, sess, dp = H.setup(w)
+    want = H.oracle_attn_full(prob, 0)
+    for B in (w.B, 5, 11, w.B):
+        out = torch.full((B, w.Hq, w.d), float("nan"), dtype=sess.dtype, device=sess.device)
+        sess.decode_attn(0, dp.q[0][:B], dp.page_table[:B], dp.seq_lens[:B], out, B=B)
+        torch.cuda.synchronize()
+        err = H.rel_err(H.to_f64(out), want[:B])
+        assert err <= H.TOL[w.dtype], (B, err)
+    assert sess.read_status() == 0
+    _free()

@@ -172,8 +172,10 @@ size_t wm_decode_attn_workspace(const wm_config* cfg, int32_t B, int32_t max_pag
  *   workspace  device, >= wm_decode_attn_workspace(cfg, B, max_pages) bytes,
  *              256-byte aligned.  It must be zero-filled before its first
  *              use; every call leaves it ready for the next one (zero-fill it
- *              again after a call that reported WM_ERR_TIMEOUT).  Calls that
- *              share a workspace must not overlap on the GPU.
+ *              again after a call that reported WM_ERR_TIMEOUT).  One
+ *              workspace serves calls of one configuration with any B and
+ *              max_pages it is large enough for.  Calls that share a
+ *              workspace must not overlap on the GPU.
  * A bad length or page id zero-fills that output row (length) or skips the
  * page, and sets WM_ERR_BOUNDS.  B = 0 is a no-op.
  */

@@ -313,7 +313,7 @@ __global__ void __launch_bounds__(kThreads, attn_ctas_per_sm(SB, G)) decode_attn
   auto chunk_end_x = [&](int64_t c) -> int64_t { return (c + 1) * NS / nchunks; };
   auto chunk_of = [&](int64_t x) -> int64_t { return ((x + 1) * nchunks - 1) / NS; };
   const int64_t gw = (int64_t)blockIdx.x * kWarps + warp;
-  int32_t* grab_ctr = p.counters + (int64_t)B * Hkv;
+  int32_t* grab_ctr = p.counters;
   // Every warp ends with exactly one request that finds no chunk; the request
   // that is last of all resets the counter for the next launch.  A request is
   // issued one chunk ahead and its result read only when the chunk is needed.
@@ -462,7 +462,6 @@ __global__ void __launch_bounds__(kThreads, attn_ctas_per_sm(SB, G)) decode_attn
   int64_t c_chunk = gw;
   int64_t cx = chunk_begin(c_chunk), cend = chunk_end_x(c_chunk), cbeg = cx;
   Cursor cc = locate(cx, pre, B, Hkv);
-  bool piece_first = true;  // the current piece starts at its chunk's first stage
   float2 q2[G][E2];
   SoftState<T, HD, G, SB> st;
   T* outp = reinterpret_cast<T*>(p.out);
@@ -537,56 +536,54 @@ __global__ void __launch_bounds__(kThreads, attn_ctas_per_sm(SB, G)) decode_attn
       } else {
         // Records of the unit's pieces: side 1 of chunk g_first, then side 0 of
         // g_first + 1 .. g_last (consecutive).  Each warp takes its ticket
+        // (counter 1 + g_first: no other crossing unit starts in that chunk)
         // first; the one that completes the unit merges, the others publish
         // their record and then set its flag (the word after the (m, l)
         // pairs) to this call's epoch, so the merging warp never publishes its
-        // own piece.  The merger clears the flags it consumed (a CUDA graph
-        // replays a call with the same epoch).
+        // own piece.  The merger clears every flag the unit raised (a CUDA
+        // graph replays a call with the same epoch, possibly over other
+        // lengths).
         const int np = (int)(g_last - g_first + 1);
         const int j_own = (int)(c_chunk - g_first);  // this piece's record in the merge
+        int32_t* ticket = p.counters + 1 + g_first;
         const float* rec1 = p.part + (int64_t)(p.max_chunks + g_first) * REC;
         const float* rec0 = p.part + (int64_t)(g_first + 1) * REC;
         auto rec_of = [&](int j) -> const float* { return j == 0 ? rec1 : rec0 + (int64_t)(j - 1) * REC; };
         auto flag_of = [&](const float* r) -> volatile int* {
           return reinterpret_cast<volatile int*>(const_cast<float*>(r) + FLAG);
         };
-        // this piece's partial as records: its chunk's first piece -> side 0,
-        // last piece -> side 1
-        auto write_records = [&](bool raise_flags) {
-          for (int side = 0; side < 2; ++side) {
-            if ((side == 0 && !piece_first) || (side == 1 && !chunk_end)) continue;
-            float* po = p.part + ((int64_t)side * p.max_chunks + c_chunk) * REC;
-            float* pm = po + G * HD;
-            if (lane_slot == 0) {
+        // this piece's partial as the one record the merge reads: the unit's
+        // first piece ends chunk g_first (side 1), every later piece starts
+        // its chunk (side 0)
+        auto write_record = [&](bool raise_flags) {
+          float* po = const_cast<float*>(rec_of(j_own));
+          float* pm = po + G * HD;
+          if (lane_slot == 0) {
 #pragma unroll
-              for (int g = 0; g < G; ++g)
+            for (int g = 0; g < G; ++g)
 #pragma unroll
-                for (int v = 0; v < SH::NVL; ++v)
+              for (int v = 0; v < SH::NVL; ++v)
 #pragma unroll
-                  for (int i = 0; i < VEC / 2; ++i)
-                    reinterpret_cast<float2*>(po + g * HD + (v * LPS + lane_part) * VEC)[i] =
-                        st.acc[g][v * VEC / 2 + i];
-            }
-            if (lane == 0) {
+                for (int i = 0; i < VEC / 2; ++i)
+                  reinterpret_cast<float2*>(po + g * HD + (v * LPS + lane_part) * VEC)[i] =
+                      st.acc[g][v * VEC / 2 + i];
+          }
+          if (lane == 0) {
 #pragma unroll
-              for (int g = 0; g < G; ++g) {
-                pm[2 * g] = st.m[g];
-                pm[2 * g + 1] = st.l[g];
-              }
+            for (int g = 0; g < G; ++g) {
+              pm[2 * g] = st.m[g];
+              pm[2 * g + 1] = st.l[g];
             }
           }
           __threadfence();
           __syncwarp();
-          if (raise_flags && lane == 0) {
-            if (piece_first) *flag_of(p.part + (int64_t)c_chunk * REC) = p.epoch;
-            if (chunk_end) *flag_of(p.part + ((int64_t)p.max_chunks + c_chunk) * REC) = p.epoch;
-          }
+          if (raise_flags && lane == 0) *flag_of(rec_of(j_own)) = p.epoch;
         };
         int last = 0;
-        if (lane == 0) last = atomicAdd(&p.counters[cc.b * Hkv + cc.h], 1) == np - 1;
+        if (lane == 0) last = atomicAdd(ticket, 1) == np - 1;
         last = __shfl_sync(FULLMASK, last, 0);
         if (!last) {
-          write_records(true);
+          write_record(true);
         } else {
           // every other piece has its ticket and only has its stores left:
           // wait (bounded) for their flags
@@ -706,7 +703,7 @@ __global__ void __launch_bounds__(kThreads, attn_ctas_per_sm(SB, G)) decode_attn
             } else {
               // stages in flight: the same batches, straight from global memory
               // (this warp's own records first, for its other lanes to read)
-              write_records(false);
+              write_record(false);
               for (int g = 0; g < G; ++g) {
                 float M = -INFINITY, Ls = 0.f;
                 float o[HD / 32];
@@ -752,11 +749,10 @@ __global__ void __launch_bounds__(kThreads, attn_ctas_per_sm(SB, G)) decode_attn
             // ready for the next launch: flags down, ticket counter zero
             for (int j = lane; j < np; j += 32)
               if (j != j_own) *flag_of(rec_of(j)) = 0;
-            if (lane == 0) p.counters[cc.b * Hkv + cc.h] = 0;
+            if (lane == 0) *ticket = 0;
           }
         }
       }
-      piece_first = false;
     }
     if (chunk_end) {  // continue with the chunk the producer moved on to
       if (chunk_for_consumer < 0) producer_step();  // a chunk shorter than the ring
@@ -766,7 +762,6 @@ __global__ void __launch_bounds__(kThreads, attn_ctas_per_sm(SB, G)) decode_attn
       cend = chunk_end_x(c_chunk);
       cbeg = cx;
       cc = locate(cx, pre, B, Hkv);
-      piece_first = true;
     } else {
       ++cx;
       advance(cc, pre, B, Hkv);

@@ -17,10 +17,12 @@ struct AttnParams {
   const int32_t* page_table;
   const int32_t* seq_lens;
   float* part;            // [2][max_chunks] records of attn_part_rec(G, d) floats: the
-                          // first / last piece partial of each chunk ([G][d] unnormalised
-                          // outputs, (max, sum) per query head in log2 units, then a
-                          // published flag, zero between launches)
-  int32_t* counters;      // [B*Hkv] arrival tickets + 1 chunk counter, zero between launches
+                          // partial of the first piece (side 0) / last piece (side 1) of
+                          // each chunk that belongs to a unit crossing a chunk boundary
+                          // ([G][d] unnormalised outputs, (max, sum) per query head in
+                          // log2 units, then a published flag, zero between launches)
+  int32_t* counters;      // [0]: chunk counter; [1 + g]: arrival tickets of the unit whose
+                          // first piece ends chunk g; zero between launches
   int32_t* status;
   int64_t page_stride;    // elements between consecutive physical pages
   int32_t B, Hq, Hkv, P, log2P, num_pages, max_pages;

@@ -60,6 +60,16 @@ constexpr int kAttnMinChunkStages = 4;  // > the per-warp ring depth
 // measured as well: the same time on the paper's 38 MB layer).
 constexpr int kAttnMinStagesPerWarp = 4;
 
+// Most work chunks any launch on this device can cut: a full grid of warps
+// (at most attn_ctas_per_sm(4096, 1) = 4 CTAs per SM) times kAttnChunksPerWarp.
+// A static split has at most one chunk per warp; a dynamic one chunks of
+// ceil(NS / (warps * kAttnChunksPerWarp)) stages or more, so at most
+// warps * kAttnChunksPerWarp of them.
+int64_t attn_chunk_capacity() {
+  return (int64_t)sm_count() * wm::attn_ctas_per_sm(4096, 1) * wm::attn_warps_per_cta() *
+         kAttnChunksPerWarp;
+}
+
 AttnPlan attn_plan(const wm_config& c, int32_t B, int32_t max_pages) {
   AttnPlan pl{};
   const int64_t max_slots = (int64_t)max_pages * c.page_size;
@@ -87,12 +97,16 @@ AttnPlan attn_plan(const wm_config& c, int32_t B, int32_t max_pages) {
     pl.chunk_stages = 0;        // static: the kernel sizes one chunk per warp
     pl.max_chunks = pl.nwarps;  // at most one chunk per warp
   }
+  // The counters sit first, at a size that depends only on the device, so a
+  // workspace that served one call still has zeros where any later call (any
+  // B, max_pages or shape) looks for its counters; the records after them
+  // need no initial value (their flags carry the call's epoch).
   const int G = c.Hq / c.Hkv;
   size_t off = 0;
+  pl.off_counters = off;
+  off += align256(sizeof(int32_t) * (1 + (size_t)attn_chunk_capacity()));
   pl.off_part = off;
   off += align256(sizeof(float) * 2 * (size_t)pl.max_chunks * wm::attn_part_rec(G, c.d));
-  pl.off_counters = off;
-  off += align256(sizeof(int32_t) * ((size_t)B * c.Hkv + 1));
   pl.total = off;
   return pl;
 }
@@ -207,6 +221,7 @@ wm_status wm_decode_attn_flags(const wm_config* c, const wm_cache* cache, int32_
   if (!aligned(q, 16) || !aligned(out, 16) || !aligned(workspace, 256)) return WM_ERR_INVALID_ARG;
   const AttnPlan pl = attn_plan(*c, B, max_pages);
   if (ws_bytes < pl.total) return WM_ERR_INVALID_ARG;
+  if (pl.max_chunks > attn_chunk_capacity()) return WM_ERR_UNSUPPORTED;  // cannot happen
 
   const int chan = c->chan_of_layer[layer];
   const size_t esz = elem_size(c->dtype);
@@ -424,8 +439,8 @@ extern "C" wm_status wm_decode_attn_noalloc(const wm_config* c, const wm_cache* 
   if (pl.total > (size_t)WM_NOALLOC_SCRATCH_BYTES) return WM_ERR_UNSUPPORTED;
   void* scratch = nullptr;
   if ((st = noalloc_scratch(&scratch)) != WM_OK) return st;
-  // the arrival tickets must start at zero; the array keeps the last call's bytes
-  if (cudaMemsetAsync((char*)scratch + pl.off_counters, 0, pl.total - pl.off_counters,
+  // the counters must start at zero; the array keeps the last call's bytes
+  if (cudaMemsetAsync((char*)scratch + pl.off_counters, 0, pl.off_part - pl.off_counters,
                       (cudaStream_t)stream) != cudaSuccess)
     return WM_ERR_CUDA;
   return wm_decode_attn(c, cache, layer, q, page_table, seq_lens, B, max_pages, out, scratch,

@@ -8,6 +8,7 @@ import numpy as np
 import pytest
 import torch
 
+from oracle import oracle as O
 from wm_synth import configs, device
 from wm_synth.inputs import make_problem
 
@@ -245,6 +246,39 @@ def test_inputs_ready_chain_matches_default_launches(name, overrides):
         assert torch.equal(outs[l], ref[l]), l
     if name == "no_compression":
         assert H.rel_err(H.to_f64(outs[3]), H.oracle_attn_full(prob, 3)) <= H.TOL[w.dtype]
+    _free()
+
+
+def test_graph_replay_over_changing_lengths():
+    """A decode loop replays one captured launch while the lengths change
+    underneath it (the replay keeps the call's epoch): the chunk layout moves
+    with the lengths, and no flag or ticket left by an earlier replay passes
+    for this replay's records."""
+    w = configs.get("no_compression").with_(L=2, k=2)
+    prob, sess, dp = H.setup(w)
+    lens = dp.seq_lens.clone()
+    out = torch.empty((w.B, w.Hq, w.d), dtype=sess.dtype, device=sess.device)
+    sess.decode_attn(0, dp.q[0], dp.page_table, lens, out)  # warm-up outside capture
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        sess.decode_attn(0, dp.q[0], dp.page_table, lens, out)
+    rng = np.random.default_rng(3)
+    full = np.asarray(prob.seq_lens, np.int64)
+    sets = [full, np.maximum(1, full // 3), rng.integers(1, full + 1), full - 17,
+            rng.integers(1, full + 1), full]
+    for S in sets:
+        lens.copy_(torch.as_tensor(S, dtype=torch.int32))
+        out.fill_(float("nan"))
+        g.replay()
+        torch.cuda.synchronize()
+        want = O.decode_attn(prob.host("q")[0], prob.host("k_pool"), prob.host("v_pool"),
+                             prob.page_table, S.astype(np.int32), chan=prob.chan[0], Hq=w.Hq,
+                             Hkv=w.Hkv, d=w.d, P=w.page, nthreads=8)
+        err = H.rel_err(H.to_f64(out), want)
+        assert err <= H.TOL[w.dtype], (S[:4], err)
+    assert sess.read_status() == 0
+    del g
     _free()
 
 

@@ -177,7 +177,8 @@ size_t wm_decode_attn_workspace(const wm_config* cfg, int32_t B, int32_t max_pag
  *              max_pages it is large enough for.  Calls that share a
  *              workspace must not overlap on the GPU.
  * A bad length or page id zero-fills that output row (length) or skips the
- * page, and sets WM_ERR_BOUNDS.  B = 0 is a no-op.
+ * page, and sets WM_ERR_BOUNDS.  B = 0 is a no-op; B above 4096 or B * Hq
+ * above 2^30 returns WM_ERR_UNSUPPORTED.
  */
 wm_status wm_decode_attn(const wm_config* cfg, const wm_cache* cache, int32_t layer,
                          const void* q, const int32_t* page_table, const int32_t* seq_lens,
@@ -194,11 +195,13 @@ wm_status wm_decode_attn(const wm_config* cfg, const wm_cache* cache, int32_t la
  * waits for it before reading anything that work may have written.
  *   WM_ATTN_INPUTS_READY: the caller promises that the work immediately
  *     before this call on `stream` writes none of the cache pools, the page
- *     table, seq_lens and the workspace (it may write q).  The kernel then
- *     starts fetching K/V while that work finishes and waits for it only
- *     before reading q.  Within one decode step this holds for layers
- *     1..L-1; it does NOT hold for the first layer after wm_kv_mix or after
- *     any update of seq_lens / the page table.
+ *     table and seq_lens (it may write q, out and this workspace: the kernel
+ *     touches those only after the wait).  The kernel then starts fetching
+ *     K/V while that work finishes and waits for it only before reading q.
+ *     Within one decode step this holds for layers 1..L-1 (the previous
+ *     layer's attention may share the workspace); it does NOT hold for the
+ *     first layer after wm_kv_mix or after any update of seq_lens / the page
+ *     table.
  * Unknown flag bits return WM_ERR_INVALID_ARG.
  */
 wm_status wm_decode_attn_flags(const wm_config* cfg, const wm_cache* cache, int32_t layer,

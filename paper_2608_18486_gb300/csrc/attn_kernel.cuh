@@ -24,12 +24,16 @@
 //    to the output.  Only units that cross a chunk boundary leave partials
 //    (at most two per chunk: its first and its last piece).  A warp takes
 //    its ticket on the unit first: the warp that completes the unit merges,
-//    every other one publishes its partial and then flags it, so the merger
-//    never publishes its own piece and waits (bounded) only for flags that
-//    are in flight.  When the merger has no stage left in flight, its idle
-//    ring receives the unit's partial records with bulk copies (one round
-//    trip for up to a ring's worth), and the merge reads them from shared
-//    memory.
+//    every other one publishes its partial and then flags it (a release
+//    store), so the merger never publishes its own piece and waits (bounded)
+//    only for flags that are in flight.  A piece that ends in the middle of
+//    its warp's chunk stores its record and takes its ticket without
+//    waiting for either, and raises its flag (or merges, if it was last)
+//    after the next stage: the warp keeps streaming instead of stalling on
+//    two round trips at every unit boundary.  When the merger has no stage
+//    left in flight, its idle ring receives the unit's partial records with
+//    bulk copies (one round trip for up to a ring's worth), and the merge
+//    reads them from shared memory.
 #include <math.h>
 
 #include "common.cuh"
@@ -111,9 +115,14 @@ __device__ __forceinline__ Cursor locate(int64_t x, const int* pre, int B, int H
   Cursor c;
   c.b = lo;
   c.nst = pre[lo + 1] - pre[lo];
-  const int64_t r = x - (int64_t)Hkv * pre[lo];
-  c.h = (int)(r / c.nst);
-  c.st = (int)(r % c.nst);
+  const int64_t r = x - (int64_t)Hkv * pre[lo];  // < Hkv * nst
+  if (r <= INT32_MAX) {
+    c.h = (int)((uint32_t)r / (uint32_t)c.nst);
+    c.st = (int)((uint32_t)r - (uint32_t)c.h * (uint32_t)c.nst);
+  } else {
+    c.h = (int)(r / c.nst);
+    c.st = (int)(r % c.nst);
+  }
   return c;
 }
 
@@ -309,9 +318,16 @@ __global__ void __launch_bounds__(kThreads, attn_ctas_per_sm(SB, G)) decode_attn
   const int64_t CH = dynamic ? p.chunk_stages : (int64_t)kWStages + 1;
   int64_t nchunks = NS / CH > 1 ? NS / CH : 1;
   if (!dynamic && nchunks > GW) nchunks = GW;
-  auto chunk_begin = [&](int64_t c) -> int64_t { return c * NS / nchunks; };
-  auto chunk_end_x = [&](int64_t c) -> int64_t { return (c + 1) * NS / nchunks; };
-  auto chunk_of = [&](int64_t x) -> int64_t { return ((x + 1) * nchunks - 1) / NS; };
+  // (32-bit division whenever the products fit: most launches)
+  const bool narrow = (NS + 1) * nchunks < (int64_t)UINT32_MAX;
+  auto chunk_begin = [&](int64_t c) -> int64_t {
+    return narrow ? (int64_t)((uint32_t)(c * NS) / (uint32_t)nchunks) : c * NS / nchunks;
+  };
+  auto chunk_end_x = [&](int64_t c) -> int64_t { return chunk_begin(c + 1); };
+  auto chunk_of = [&](int64_t x) -> int64_t {
+    const int64_t t = (x + 1) * nchunks - 1;
+    return narrow ? (int64_t)((uint32_t)t / (uint32_t)NS) : t / NS;
+  };
   const int64_t gw = (int64_t)blockIdx.x * kWarps + warp;
   int32_t* grab_ctr = p.counters;
   // Every warp ends with exactly one request that finds no chunk; the request
@@ -465,6 +481,109 @@ __global__ void __launch_bounds__(kThreads, attn_ctas_per_sm(SB, G)) decode_attn
   float2 q2[G][E2];
   SoftState<T, HD, G, SB> st;
   T* outp = reinterpret_cast<T*>(p.out);
+
+  // ---- partial records of units that cross chunk boundaries.  The records
+  // of a unit whose first piece ends chunk gf: side 1 of chunk gf, then
+  // side 0 of chunks gf + 1, gf + 2, ... (consecutive).  Each piece takes its
+  // ticket (counter 1 + gf: no other crossing unit starts in chunk gf) before
+  // its flag goes up; the piece completing the unit merges, every other one
+  // publishes its record and then sets the record's flag (the word after the
+  // (m, l) pairs) to this call's epoch, so the merging warp never publishes
+  // its own piece.  The merger clears every flag the unit raised and the
+  // ticket (a CUDA graph replays a call with the same epoch, possibly over
+  // other lengths).
+  auto rec_at = [&](int gf, int j) -> float* {
+    return p.part + (j == 0 ? (int64_t)(p.max_chunks + gf) : (int64_t)(gf + j)) * REC;
+  };
+  auto flag_at = [&](float* r) -> int* { return reinterpret_cast<int*>(r + FLAG); };
+  // this warp's merged piece (registers) as a record
+  auto store_record = [&](float* po) {
+    float* pm = po + G * HD;
+    if (lane_slot == 0) {
+#pragma unroll
+      for (int g = 0; g < G; ++g)
+#pragma unroll
+        for (int v = 0; v < SH::NVL; ++v)
+#pragma unroll
+          for (int i = 0; i < VEC / 2; ++i)
+            reinterpret_cast<float2*>(po + g * HD + (v * LPS + lane_part) * VEC)[i] =
+                st.acc[g][v * VEC / 2 + i];
+    }
+    if (lane == 0) {
+#pragma unroll
+      for (int g = 0; g < G; ++g) {
+        pm[2 * g] = st.m[g];
+        pm[2 * g + 1] = st.l[g];
+      }
+    }
+  };
+  // every other piece has its ticket and at most its stores left: wait
+  // (bounded) for their flags; false (and WM_ERR_TIMEOUT) if one never came
+  auto wait_flags = [&](int gf, int np, int j_own) -> bool {
+    bool ready = false;
+    const uint64_t t0 = globaltimer_ns();
+    for (uint32_t it = 0;; ++it) {
+      bool mine = true;
+      for (int j = lane; j < np; j += 32)
+        if (j != j_own) mine = mine && (ld_acquire_gpu(flag_at(rec_at(gf, j))) == p.epoch);
+      ready = __all_sync(FULLMASK, mine);
+      if (ready || ((it & 63u) == 63u && globaltimer_ns() - t0 > kWaitLimitNs)) break;
+    }
+    if (!ready && lane == 0) report(p.status, WM_ERR_TIMEOUT);
+    __syncwarp();  // every lane's acquire precedes the whole warp's reads
+    return ready;
+  };
+  // merge all np records of the unit from global memory into its output rows
+  auto merge_global = [&](int gf, int np, int rowbase) {
+    for (int g = 0; g < G; ++g) {
+      float M = -INFINITY, Ls = 0.f;
+      float o[HD / 32];
+#pragma unroll
+      for (int i = 0; i < HD / 32; ++i) o[i] = 0.f;
+      for (int r0 = 0; r0 < np; r0 += MB) {
+        float mq[MB], lq[MB], ov[MB][HD / 32];
+#pragma unroll
+        for (int jb = 0; jb < MB; ++jb) {
+          const int j = r0 + jb;
+          const bool in = j < np;
+          const float* rj = rec_at(gf, j);
+          mq[jb] = in ? __ldcg(rj + G * HD + 2 * g) : -INFINITY;
+          lq[jb] = in ? __ldcg(rj + G * HD + 2 * g + 1) : 0.f;
+#pragma unroll
+          for (int i = 0; i < HD / 32; ++i)
+            ov[jb][i] = in ? __ldcg(rj + g * HD + lane + 32 * i) : 0.f;
+        }
+        float Mn = M;
+#pragma unroll
+        for (int jb = 0; jb < MB; ++jb) Mn = fmaxf(Mn, mq[jb]);
+        if (Mn == -INFINITY) continue;
+        const float rescale = exp2f(M - Mn);  // 0 on the first batch
+        Ls *= rescale;
+#pragma unroll
+        for (int i = 0; i < HD / 32; ++i) o[i] *= rescale;
+#pragma unroll
+        for (int jb = 0; jb < MB; ++jb) {
+          if (mq[jb] == -INFINITY) continue;
+          const float w = exp2f(mq[jb] - Mn);
+          Ls = fmaf(w, lq[jb], Ls);
+#pragma unroll
+          for (int i = 0; i < HD / 32; ++i) o[i] = fmaf(w, ov[jb][i], o[i]);
+        }
+        M = Mn;
+      }
+      const float inv = Ls > 0.f ? 1.f / Ls : 0.f;
+#pragma unroll
+      for (int i = 0; i < HD / 32; ++i)
+        outp[((int64_t)rowbase + g) * HD + lane + 32 * i] = Elem<T>::from_f(o[i] * inv);
+    }
+  };
+  // ready for the next launch: flags down, ticket counter zero
+  auto release_unit = [&](int gf, int np, int j_own) {
+    for (int j = lane; j < np; j += 32)
+      if (j != j_own) *reinterpret_cast<volatile int*>(flag_at(rec_at(gf, j))) = 0;
+    if (lane == 0) p.counters[1 + gf] = 0;
+  };
+  int pend_np = 0, pend_tk = 0, pend_g = 0, pend_row = 0;  // a piece awaiting its flag
   for (uint32_t seq = 0;; ++seq) {
     const int buf = (int)(seq % kWStages);
     bool ok = mbar_wait(&bars[warp][buf], (seq / kWStages) & 1);
@@ -490,6 +609,18 @@ __global__ void __launch_bounds__(kThreads, attn_ctas_per_sm(SB, G)) decode_attn
         for (int i = 0; i < E2; ++i) st.acc[g][i] = make_float2(0.f, 0.f);
       }
     }
+    // A stage that ends a piece of a unit crossing chunk boundaries takes the
+    // piece's ticket before its math, so the atomic's round trip overlaps it.
+    const bool chunk_end = (cx == cend - 1);
+    const bool piece_end = chunk_end || cc.st == cc.nst - 1;
+    int64_t g_first = 0, g_last = 0;
+    int tk = 0;
+    if (piece_end) {
+      const int64_t U = (int64_t)Hkv * pre[cc.b] + (int64_t)cc.h * cc.nst;
+      g_first = chunk_of(U);
+      g_last = chunk_of(U + cc.nst - 1);
+      if (g_first != g_last && lane == 0) tk = atomicAdd(p.counters + 1 + g_first, 1);
+    }
     const int valid_slots = lens[cc.b] - cc.st * STAGE_SLOTS;
     const uint64_t mask = masks[warp][buf];
     const T* Ks = myring + buf * 2 * STAGE_ELEMS;
@@ -503,8 +634,20 @@ __global__ void __launch_bounds__(kThreads, attn_ctas_per_sm(SB, G)) decode_attn
     __syncwarp();  // every lane is done with this ring slot
     producer_step();
 
-    const bool chunk_end = (cx == cend - 1);
-    if (chunk_end || cc.st == cc.nst - 1) {
+    if (pend_np > 0) {
+      // the piece that ended one stage ago, in the middle of this chunk: its
+      // record and ticket went out then; its stores have landed by now
+      const bool last = __shfl_sync(FULLMASK, pend_tk, 0) == pend_np - 1;
+      if (!last) {
+        __syncwarp();
+        if (lane == 0) st_release_gpu(flag_at(rec_at(pend_g, pend_np - 1)), p.epoch);
+      } else if (wait_flags(pend_g, pend_np, pend_np - 1)) {
+        merge_global(pend_g, pend_np, pend_row);
+        release_unit(pend_g, pend_np, pend_np - 1);
+      }
+      pend_np = 0;
+    }
+    if (piece_end) {
       // merge the SPW lane groups of the warp
 #pragma unroll
       for (int g = 0; g < G; ++g) {
@@ -528,78 +671,30 @@ __global__ void __launch_bounds__(kThreads, attn_ctas_per_sm(SB, G)) decode_attn
         st.m[g] = M;
         st.l[g] = Ls;
       }
-      const int64_t rowbase = (int64_t)cc.b * p.Hq + cc.h * G;
-      const int64_t U = (int64_t)Hkv * pre[cc.b] + (int64_t)cc.h * cc.nst;
-      const int64_t g_first = chunk_of(U), g_last = chunk_of(U + cc.nst - 1);
+      const int rowbase = cc.b * p.Hq + cc.h * G;
       if (g_first == g_last) {
-        if (lane_slot == 0) write_rows<T, HD, G, SB>(outp + rowbase * HD, lane_part, st);
+        if (lane_slot == 0) write_rows<T, HD, G, SB>(outp + (int64_t)rowbase * HD, lane_part, st);
       } else {
-        // Records of the unit's pieces: side 1 of chunk g_first, then side 0 of
-        // g_first + 1 .. g_last (consecutive).  Each warp takes its ticket
-        // (counter 1 + g_first: no other crossing unit starts in that chunk)
-        // first; the one that completes the unit merges, the others publish
-        // their record and then set its flag (the word after the (m, l)
-        // pairs) to this call's epoch, so the merging warp never publishes its
-        // own piece.  The merger clears every flag the unit raised (a CUDA
-        // graph replays a call with the same epoch, possibly over other
-        // lengths).
+        const int gf = (int)g_first;
         const int np = (int)(g_last - g_first + 1);
         const int j_own = (int)(c_chunk - g_first);  // this piece's record in the merge
-        int32_t* ticket = p.counters + 1 + g_first;
-        const float* rec1 = p.part + (int64_t)(p.max_chunks + g_first) * REC;
-        const float* rec0 = p.part + (int64_t)(g_first + 1) * REC;
-        auto rec_of = [&](int j) -> const float* { return j == 0 ? rec1 : rec0 + (int64_t)(j - 1) * REC; };
-        auto flag_of = [&](const float* r) -> volatile int* {
-          return reinterpret_cast<volatile int*>(const_cast<float*>(r) + FLAG);
-        };
-        // this piece's partial as the one record the merge reads: the unit's
-        // first piece ends chunk g_first (side 1), every later piece starts
-        // its chunk (side 0)
-        auto write_record = [&](bool raise_flags) {
-          float* po = const_cast<float*>(rec_of(j_own));
-          float* pm = po + G * HD;
-          if (lane_slot == 0) {
-#pragma unroll
-            for (int g = 0; g < G; ++g)
-#pragma unroll
-              for (int v = 0; v < SH::NVL; ++v)
-#pragma unroll
-                for (int i = 0; i < VEC / 2; ++i)
-                  reinterpret_cast<float2*>(po + g * HD + (v * LPS + lane_part) * VEC)[i] =
-                      st.acc[g][v * VEC / 2 + i];
-          }
-          if (lane == 0) {
-#pragma unroll
-            for (int g = 0; g < G; ++g) {
-              pm[2 * g] = st.m[g];
-              pm[2 * g + 1] = st.l[g];
-            }
-          }
-          __threadfence();
-          __syncwarp();
-          if (raise_flags && lane == 0) *flag_of(rec_of(j_own)) = p.epoch;
-        };
-        int last = 0;
-        if (lane == 0) last = atomicAdd(ticket, 1) == np - 1;
-        last = __shfl_sync(FULLMASK, last, 0);
-        if (!last) {
-          write_record(true);
+        if (!chunk_end) {
+          // The unit ends here and the chunk goes on (so this is the unit's
+          // last piece, j_own = np - 1): store the record now, read the
+          // ticket and raise the flag after the next stage instead of
+          // stalling on both round trips in the middle of the stream.
+          store_record(rec_at(gf, j_own));
+          pend_tk = tk;
+          pend_np = np;
+          pend_g = gf;
+          pend_row = rowbase;
         } else {
-          // every other piece has its ticket and only has its stores left:
-          // wait (bounded) for their flags
-          bool ready = false;
-          const uint64_t t0 = globaltimer_ns();
-          for (uint32_t it = 0;; ++it) {
-            bool mine = true;
-            for (int j = lane; j < np; j += 32)
-              if (j != j_own) mine = mine && (*flag_of(rec_of(j)) == p.epoch);
-            ready = __all_sync(FULLMASK, mine);
-            if (ready || ((it & 63u) == 63u && globaltimer_ns() - t0 > kWaitLimitNs)) break;
-          }
-          if (!ready) {
-            if (lane == 0) report(p.status, WM_ERR_TIMEOUT);
-          } else {
-            __threadfence();
+          const bool last = __shfl_sync(FULLMASK, tk, 0) == np - 1;
+          if (!last) {
+            store_record(rec_at(gf, j_own));
+            __syncwarp();
+            if (lane == 0) st_release_gpu(flag_at(rec_at(gf, j_own)), p.epoch);
+          } else if (wait_flags(gf, np, j_own)) {
             if (p_done && seq + 1 == pseq) {
               // no stage in flight: the ring takes ROUND records per round
               float* rs = reinterpret_cast<float*>(myring);
@@ -620,10 +715,10 @@ __global__ void __launch_bounds__(kThreads, attn_ctas_per_sm(SB, G)) decode_attn
                 if (lane == 0) {
                   mbar_arrive_expect_tx(&qbars[warp], (uint32_t)n * RB);
                   if (r0 == 0) {
-                    bulk_g2s(rs, rec1, RB, &qbars[warp], policy);
-                    if (n > 1) bulk_g2s(rs + REC, rec0, (uint32_t)(n - 1) * RB, &qbars[warp], policy);
+                    bulk_g2s(rs, rec_at(gf, 0), RB, &qbars[warp], policy);
+                    if (n > 1) bulk_g2s(rs + REC, rec_at(gf, 1), (uint32_t)(n - 1) * RB, &qbars[warp], policy);
                   } else {
-                    bulk_g2s(rs, rec0 + (int64_t)(r0 - 1) * REC, (uint32_t)n * RB, &qbars[warp], policy);
+                    bulk_g2s(rs, rec_at(gf, r0), (uint32_t)n * RB, &qbars[warp], policy);
                   }
                 }
                 // qbars completed phase 0 with the first query; round r is phase r + 1
@@ -697,59 +792,18 @@ __global__ void __launch_bounds__(kThreads, attn_ctas_per_sm(SB, G)) decode_attn
                   const float inv = Ls[g] > 0.f ? 1.f / Ls[g] : 0.f;
 #pragma unroll
                   for (int i = 0; i < HD / 32; ++i)
-                    outp[(rowbase + g) * HD + lane + 32 * i] = Elem<T>::from_f(o[g][i] * inv);
+                    outp[((int64_t)rowbase + g) * HD + lane + 32 * i] = Elem<T>::from_f(o[g][i] * inv);
                 }
               }
             } else {
-              // stages in flight: the same batches, straight from global memory
-              // (this warp's own records first, for its other lanes to read)
-              write_record(false);
-              for (int g = 0; g < G; ++g) {
-                float M = -INFINITY, Ls = 0.f;
-                float o[HD / 32];
-#pragma unroll
-                for (int i = 0; i < HD / 32; ++i) o[i] = 0.f;
-                for (int r0 = 0; r0 < np; r0 += MB) {
-                  float mq[MB], lq[MB], ov[MB][HD / 32];
-#pragma unroll
-                  for (int jb = 0; jb < MB; ++jb) {
-                    const int j = r0 + jb;
-                    const bool in = j < np;
-                    const float* rj = j == 0 ? rec1 : rec0 + (int64_t)(j - 1) * REC;
-                    mq[jb] = in ? __ldcg(rj + G * HD + 2 * g) : -INFINITY;
-                    lq[jb] = in ? __ldcg(rj + G * HD + 2 * g + 1) : 0.f;
-#pragma unroll
-                    for (int i = 0; i < HD / 32; ++i)
-                      ov[jb][i] = in ? __ldcg(rj + g * HD + lane + 32 * i) : 0.f;
-                  }
-                  float Mn = M;
-#pragma unroll
-                  for (int jb = 0; jb < MB; ++jb) Mn = fmaxf(Mn, mq[jb]);
-                  if (Mn == -INFINITY) continue;
-                  const float rescale = exp2f(M - Mn);  // 0 on the first batch
-                  Ls *= rescale;
-#pragma unroll
-                  for (int i = 0; i < HD / 32; ++i) o[i] *= rescale;
-#pragma unroll
-                  for (int jb = 0; jb < MB; ++jb) {
-                    if (mq[jb] == -INFINITY) continue;
-                    const float w = exp2f(mq[jb] - Mn);
-                    Ls = fmaf(w, lq[jb], Ls);
-#pragma unroll
-                    for (int i = 0; i < HD / 32; ++i) o[i] = fmaf(w, ov[jb][i], o[i]);
-                  }
-                  M = Mn;
-                }
-                const float inv = Ls > 0.f ? 1.f / Ls : 0.f;
-#pragma unroll
-                for (int i = 0; i < HD / 32; ++i)
-                  outp[(rowbase + g) * HD + lane + 32 * i] = Elem<T>::from_f(o[i] * inv);
-              }
+              // stages in flight: the same batches, straight from global
+              // memory (this warp's own record first, for its other lanes)
+              store_record(rec_at(gf, j_own));
+              __threadfence();
+              __syncwarp();
+              merge_global(gf, np, rowbase);
             }
-            // ready for the next launch: flags down, ticket counter zero
-            for (int j = lane; j < np; j += 32)
-              if (j != j_own) *flag_of(rec_of(j)) = 0;
-            if (lane == 0) *ticket = 0;
+            release_unit(gf, np, j_own);
           }
         }
       }

@@ -217,6 +217,7 @@ wm_status wm_decode_attn_flags(const wm_config* c, const wm_cache* cache, int32_
   if ((int64_t)max_pages * c->page_size > INT32_MAX / 2) return WM_ERR_INVALID_ARG;
   if (B == 0) return WM_OK;
   if (B > kAttnMaxBatch) return WM_ERR_UNSUPPORTED;
+  if ((int64_t)B * c->Hq > INT32_MAX / 2) return WM_ERR_UNSUPPORTED;  // 32-bit output rows
   if (!q || !page_table || !seq_lens || !out || !workspace) return WM_ERR_INVALID_ARG;
   if (!aligned(q, 16) || !aligned(out, 16) || !aligned(workspace, 256)) return WM_ERR_INVALID_ARG;
   const AttnPlan pl = attn_plan(*c, B, max_pages);

@@ -28,12 +28,13 @@
 //    store), so the merger never publishes its own piece and waits (bounded)
 //    only for flags that are in flight.  A piece that ends in the middle of
 //    its warp's chunk stores its record and takes its ticket without
-//    waiting for either, and raises its flag (or merges, if it was last)
-//    after the next stage: the warp keeps streaming instead of stalling on
-//    two round trips at every unit boundary.  When the merger has no stage
-//    left in flight, its idle ring receives the unit's partial records with
-//    bulk copies (one round trip for up to a ring's worth), and the merge
-//    reads them from shared memory.
+//    waiting for either, and raises its flag (or merges, if it was last) at
+//    the chunk's end: a release or fence issued while the warp's bulk copies
+//    are in flight waits for them, which stalled the stream at every unit
+//    boundary.  Tickets are taken before the math of a piece's last stage.
+//    When the merger has no stage left in flight, its idle ring receives the
+//    unit's partial records with bulk copies (one round trip for up to a
+//    ring's worth), and the merge reads them from shared memory.
 #include <math.h>
 
 #include "common.cuh"
@@ -357,7 +358,11 @@ __global__ void __launch_bounds__(kThreads, attn_ctas_per_sm(SB, G)) decode_attn
 
   // ---- page-table window of the producer: lane i holds the page id of
   // logical page win0 + i (cur) and win0 + 32 + i (nxt) of sequence win_b.
+  // The first 64 page ids of the unit after the current one are fetched one
+  // stage before its first copy (pf_*), and nxt is read only when a stage
+  // needs it, so no page-table load sits between two copies of the stream.
   int win_b = -1, win0 = 0, pg_cur = -1, pg_nxt = -1;
+  int pf_b = -1, pf_cur = -1, pf_nxt = -1;
   auto load_pg = [&](int b, int lp) -> int {
     return lp < p.max_pages ? __ldg(p.page_table + (int64_t)b * p.max_pages + lp) : -1;
   };
@@ -366,8 +371,13 @@ __global__ void __launch_bounds__(kThreads, attn_ctas_per_sm(SB, G)) decode_attn
     if (b != win_b || lp < win0 || lp >= win0 + 64) {
       win_b = b;
       win0 = lp;
-      pg_cur = load_pg(b, lp + lane);
-      pg_nxt = load_pg(b, lp + 32 + lane);
+      if (lp == 0 && b == pf_b) {
+        pg_cur = pf_cur;
+        pg_nxt = pf_nxt;
+      } else {
+        pg_cur = load_pg(b, lp + lane);
+        pg_nxt = load_pg(b, lp + 32 + lane);
+      }
     } else if (lp >= win0 + 32) {
       win0 += 32;
       pg_cur = pg_nxt;
@@ -375,6 +385,7 @@ __global__ void __launch_bounds__(kThreads, attn_ctas_per_sm(SB, G)) decode_attn
     }
     const int idx = lp + lane_off - win0;  // 0 .. 63
     const int a = __shfl_sync(FULLMASK, pg_cur, idx & 31);
+    if (__all_sync(FULLMASK, idx < 32)) return a;
     const int c = __shfl_sync(FULLMASK, pg_nxt, idx & 31);
     return idx < 32 ? a : c;
   };
@@ -438,6 +449,11 @@ __global__ void __launch_bounds__(kThreads, attn_ctas_per_sm(SB, G)) decode_attn
     ++pseq;
     ++px;
     advance(pc, pre, B, Hkv);
+    if (pc.st == 0 && px < pend && pc.b < B && pc.b != pf_b) {  // the next copy opens a unit
+      pf_b = pc.b;
+      pf_cur = load_pg(pc.b, lane);
+      pf_nxt = load_pg(pc.b, 32 + lane);
+    }
   };
   // Issue the next stage; when the current chunk is used up, first move on
   // to the chunk requested ahead (the consumer follows through
@@ -634,9 +650,11 @@ __global__ void __launch_bounds__(kThreads, attn_ctas_per_sm(SB, G)) decode_attn
     __syncwarp();  // every lane is done with this ring slot
     producer_step();
 
-    if (pend_np > 0) {
-      // the piece that ended one stage ago, in the middle of this chunk: its
-      // record and ticket went out then; its stores have landed by now
+    if (pend_np > 0 && chunk_end) {
+      // the piece that ended in the middle of this chunk: its record and
+      // ticket went out then; its flag goes up now, where (in a static split)
+      // no copy of this warp is in flight any more -- a release issued
+      // while bulk copies are in flight waited for them
       const bool last = __shfl_sync(FULLMASK, pend_tk, 0) == pend_np - 1;
       if (!last) {
         __syncwarp();
@@ -680,9 +698,10 @@ __global__ void __launch_bounds__(kThreads, attn_ctas_per_sm(SB, G)) decode_attn
         const int j_own = (int)(c_chunk - g_first);  // this piece's record in the merge
         if (!chunk_end) {
           // The unit ends here and the chunk goes on (so this is the unit's
-          // last piece, j_own = np - 1): store the record now, read the
-          // ticket and raise the flag after the next stage instead of
-          // stalling on both round trips in the middle of the stream.
+          // last piece, j_own = np - 1; a chunk holds at most one such
+          // piece, its first): store the record now, read the ticket and
+          // raise the flag (or merge) at the chunk's end instead of stalling
+          // the stream in its middle.
           store_record(rec_at(gf, j_own));
           pend_tk = tk;
           pend_np = np;

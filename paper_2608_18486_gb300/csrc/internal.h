@@ -37,6 +37,7 @@ struct AttnParams {
 
 // Resident CTAs per SM the attention kernel is built for: 4 with 4 KB stages
 // and one query head per kv head, else 2 (GQA keeps G query rows per lane).
+// The planner uses 8 KB stages only.
 constexpr int attn_ctas_per_sm(int stage_bytes, int G) { return stage_bytes == 4096 && G == 1 ? 4 : 2; }
 
 // Floats per partial record: G*d outputs, (max, sum) per head, a "published"

@@ -43,11 +43,11 @@ struct AttnPlan {
 };
 
 constexpr int kAttnMaxBatch = 4096;
-// Launches reading less than this many KV bytes (upper bound from the page
-// table width) with one query head per kv head use 4 KB stages and 4 CTAs
-// per SM (16 warps: more latency hiding for short launches); larger ones and
-// grouped-query launches (2 CTAs per SM either way) use 8 KB stages.
-constexpr double kAttnSmallLaunchBytes = 1.0e9;
+// K + V bytes of one pipeline stage: 8 KB, 2 CTAs (8 warps) per SM.  A warp
+// spends about as long on the bookkeeping of a stage (wait, copy issue,
+// piece checks) as on its math, so 4 KB stages at 4 CTAs per SM were
+// slower (24.0 vs 21.0 us on a 100 MB launch measured side by side).
+constexpr int kAttnStageBytes = 8192;
 // Launches reading at least this many KV bytes hand out work dynamically:
 // chunks of the stage stream taken from an atomic counter, about
 // kAttnChunksPerWarp per warp, so warps that stream faster take more.
@@ -61,12 +61,12 @@ constexpr int kAttnMinChunkStages = 4;  // > the per-warp ring depth
 constexpr int kAttnMinStagesPerWarp = 4;
 
 // Most work chunks any launch on this device can cut: a full grid of warps
-// (at most attn_ctas_per_sm(4096, 1) = 4 CTAs per SM) times kAttnChunksPerWarp.
+// (attn_ctas_per_sm CTAs per SM) times kAttnChunksPerWarp.
 // A static split has at most one chunk per warp; a dynamic one chunks of
 // ceil(NS / (warps * kAttnChunksPerWarp)) stages or more, so at most
 // warps * kAttnChunksPerWarp of them.
 int64_t attn_chunk_capacity() {
-  return (int64_t)sm_count() * wm::attn_ctas_per_sm(4096, 1) * wm::attn_warps_per_cta() *
+  return (int64_t)sm_count() * wm::attn_ctas_per_sm(kAttnStageBytes, 1) * wm::attn_warps_per_cta() *
          kAttnChunksPerWarp;
 }
 
@@ -74,7 +74,7 @@ AttnPlan attn_plan(const wm_config& c, int32_t B, int32_t max_pages) {
   AttnPlan pl{};
   const int64_t max_slots = (int64_t)max_pages * c.page_size;
   const double kv_bytes = (double)B * c.Hkv * max_slots * 2.0 * c.d * elem_size(c.dtype);
-  pl.stage_bytes = (kv_bytes < kAttnSmallLaunchBytes && c.Hq == c.Hkv) ? 4096 : 8192;
+  pl.stage_bytes = kAttnStageBytes;
   const int ctas_per_sm = wm::attn_ctas_per_sm(pl.stage_bytes, c.Hq / c.Hkv);
   const int stage = wm::attn_stage_slots(pl.stage_bytes, c.dtype, c.d);
   const int64_t ns_max = (int64_t)B * c.Hkv * ((max_slots + stage - 1) / stage);

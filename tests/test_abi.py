@@ -96,6 +96,27 @@ def test_compute_calls_reject_bad_arguments_before_launching():
     assert W.wm_kv_mix(c, cache, wts, None, None, None, 0, 4, None, 0, None, None) == W.WM_OK
 
 
+def test_attention_refuses_output_rows_past_32_bits_before_launching():
+    # 4096 sequences x 2^19 query heads: more output rows than the kernel's
+    # 32-bit row index covers
+    c = cfg(Hq=1 << 19, Hkv=1 << 16)
+    assert W.wm_config_check(c) == W.WM_OK
+    n = W.wm_cache_bytes(c, 1)
+    cache = W.wm_cache_alloc(c, 1 << 40, n, 1)
+    fake = 1 << 41
+    ws = W.wm_decode_attn_workspace(c, 4096, 1)
+    assert W.wm_decode_attn(c, cache, 0, fake, fake, fake, 4096, 1, fake, fake, ws, None,
+                            None) == W.WM_ERR_UNSUPPORTED
+
+
+def test_attention_workspace_grows_with_the_batch():
+    # a workspace sized for the largest batch serves every smaller one
+    c = cfg()
+    sizes = [W.wm_decode_attn_workspace(c, b, 513) for b in (1, 2, 5, 16, 32, 100, 1000, 4096)]
+    assert all(a <= b for a, b in zip(sizes, sizes[1:])), sizes
+    assert all(s % 256 == 0 for s in sizes)
+
+
 def test_status_strings():
     for code in range(6):
         assert W.wm_status_string(code) and W.wm_status_string(code) != "unknown status"

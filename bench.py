@@ -50,7 +50,7 @@ def measured_peak():
 
 def kernel_source_hash() -> str:
     h = hashlib.sha256()
-    for f in ("attn.cu", "attn_kernel.cuh", "attn_bf16.cu", "common.cuh", "internal.h"):
+    for f in ("attn.cu", "attn_kernel.cuh", "attn_bf16.cu", "common.cuh", "internal.h", "wm_api.cu"):
         with open(os.path.join(ROOT, "paper_2608_18486_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:16]

@@ -15,7 +15,9 @@
  *    queries, outputs, cache pools, page tables, workspaces, status word).
  *    Pointers marked "device" must be device (or managed) memory of the
  *    current CUDA device.  The library allocates no memory and keeps no state
- *    between calls other than a per-device attribute cache.
+ *    between calls other than per-device attribute and address caches, a
+ *    process-wide counter that tags each attention call (its epoch), and the
+ *    fixed scratch array of wm_decode_attn_noalloc.
  *  - Streams: `stream` is a cudaStream_t (NULL = legacy default stream).
  *    Compute calls only enqueue work and return; results are valid after the
  *    stream is synchronised.

@@ -18,6 +18,10 @@ import numpy as np
 _HERE = os.path.dirname(os.path.abspath(__file__))
 SRC = os.path.join(_HERE, "wm_oracle.c")
 LIB_PATH = os.path.join(_HERE, "liboracle.so")
+# A compiled copy of the oracle to load instead of liboracle.so: the mutation
+# test (tests/test_oracle_mutants.py) points it at copies with a planted
+# mistake to show that the pins catch each one.
+ALT_LIB = os.environ.get("WM_ORACLE_LIB")
 _lib = None
 
 _dp = ctypes.POINTER(ctypes.c_double)
@@ -37,9 +41,12 @@ def build(verbose: bool = False) -> str:
 def lib():
     global _lib
     if _lib is None:
-        if not os.path.exists(LIB_PATH) or os.path.getmtime(LIB_PATH) < os.path.getmtime(SRC):
-            build()
-        L = ctypes.CDLL(LIB_PATH)
+        if ALT_LIB:
+            L = ctypes.CDLL(ALT_LIB)
+        else:
+            if not os.path.exists(LIB_PATH) or os.path.getmtime(LIB_PATH) < os.path.getmtime(SRC):
+                build()
+            L = ctypes.CDLL(LIB_PATH)
         L.orc_max_threads.restype = ctypes.c_int
         L.orc_rmsnorm.argtypes = [_dp, ctypes.c_int, ctypes.c_double, _dp, _dp]
         L.orc_rope.argtypes = [_dp, ctypes.c_int, ctypes.c_double, ctypes.c_double]

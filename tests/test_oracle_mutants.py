@@ -1,9 +1,10 @@
 """The oracle's pins catch plausible mistakes (CPU only).
 
 Each case plants one mistake in a copy of the C oracle -- a flipped RoPE
-sign, the router input stacked in the wrong order, a dropped gain or norm,
-the wrong kv head for a grouped query, a missing 1/sqrt(d), a prefill query
-reading its own slot, ... -- compiles the copy, and runs the pin suite
+sign, the router input stacked in the wrong order, a dropped gain, bias or
+norm, a transposed projection, the wrong kv head for a grouped query, a
+missing 1/sqrt(d), a prefill query reading its own slot, ... -- compiles the
+copy, and runs the pin suite
 (tests/test_oracle_pins.py) against it in a child process.  A mutant that
 passes every pin would mean a wrong oracle could go unnoticed, so each one
 must make at least one pin fail.  The unmodified copy, built the same way,
@@ -44,6 +45,12 @@ MUTANTS = [
      "o[e] += wt * rd(k_pool, base[t] + e, dt);\n    }\n    for (int e = 0; e < d; ++e) o[e] /= wsum;\n    m_attn += 2 * (int64_t)S * d;"),
     ("prefill_reads_own_slot", "int nslots = i + 1; /* slots 0 .. i */",
      "int nslots = i + 2; /* slots 0 .. i */"),
+    ("prefill_scale_missing", "s[t] = acc * scale;", "s[t] = acc;"),
+    ("router_bias_dropped", "double z = rd(br, (int64_t)X * k * L + o, dt);", "double z = 0.0;"),
+    ("router_shared_by_branches", "const void* W = adv(Wr, (int64_t)X * k * L * in_dim, dt);",
+     "const void* W = Wr;"),
+    ("projection_transposed", "acc += rd(W_Xj, n * D + e, dt) * xn[e];",
+     "acc += rd(W_Xj, (int64_t)e * n_out + n, dt) * xn[e];"),
 ]
 
 

@@ -246,6 +246,9 @@ def oracle_pool_estimate(prob, budget_s: float = 4.0, nthreads: int | None = Non
 
 
 # ---------------------------------------------------------------- arms
+REF_TOTAL_S = 120.0  # oracle seconds a whole --impl reference run may spend
+
+
 def run_reference(args, w):
     rank, world, _ = dist_env()
     if rank != 0:
@@ -254,8 +257,11 @@ def run_reference(args, w):
     prob = make_problem(w, seed=0)
     times = []
     cores, sample = None, ""
+    # every step is a bounded sample of the workload; together they stay
+    # within about REF_TOTAL_S of oracle time whatever --steps asks for
+    per_step = min(args.ref_budget, REF_TOTAL_S / max(1, args.warmup + args.steps))
     for i in range(args.warmup + args.steps):
-        t, cores, sample = oracle_step_estimate(prob, budget_s=args.ref_budget)
+        t, cores, sample = oracle_step_estimate(prob, budget_s=per_step)
         if i >= args.warmup:
             times.append(t)
     step_s = statistics.median(times)

@@ -48,3 +48,19 @@ def test_problem_paging_is_a_partition():
     w = configs.get("large")
     p = inputs.make_problem(w, seed=0)
     assert p.seq_lens.min() >= w.ctx_lo and p.seq_lens.max() <= w.ctx
+
+
+def test_chunked_generation_equals_the_one_pass_definition():
+    """values()/values_at() fill large requests in chunks on several threads;
+    every bit must equal the element-wise definition taken in one pass."""
+    n = 2 * gen._CHUNK + 12345
+    for dtype in ("f32", "bf16"):
+        one = gen.normal_f32(5, 9, np.arange(777, 777 + n, dtype=np.uint64), 0.3, -0.2)
+        one = one if dtype == "f32" else gen.f32_to_bf16_bits(one)
+        got = gen.values(dtype, 5, 9, 777, n, 0.3, -0.2)
+        assert got.dtype == one.dtype and np.array_equal(got, one)
+        idx = np.random.default_rng(1).integers(0, 2 ** 40, size=(2, n // 2)).astype(np.uint64)
+        at = gen.values_at(dtype, 5, 9, idx, 0.3, -0.2)
+        ref = gen.normal_f32(5, 9, idx, 0.3, -0.2)
+        assert at.shape == idx.shape
+        assert np.array_equal(at, ref if dtype == "f32" else gen.f32_to_bf16_bits(ref))

@@ -22,6 +22,9 @@ Definition
 """
 from __future__ import annotations
 
+import concurrent.futures as cf
+import os
+
 import numpy as np
 
 GAMMA = np.uint64(0x9E3779B97F4A7C15)
@@ -86,26 +89,55 @@ def bf16_bits_to_f32(b: np.ndarray) -> np.ndarray:
     return (np.asarray(b, dtype=np.uint16).astype(np.uint32) << np.uint32(16)).view(np.float32)
 
 
+def _stored(dtype: str, seed: int, stream: int, idx: np.ndarray, std: float,
+            mean: float) -> np.ndarray:
+    v = normal_f32(seed, stream, idx, std, mean)
+    return v if dtype == "f32" else f32_to_bf16_bits(v)
+
+
+# Large requests are cut into chunks of this many values, filled by a few
+# threads (numpy releases the GIL in its loops): the same bits as one pass,
+# without gigabyte-sized temporaries.
+_CHUNK = 1 << 20
+
+
+def _chunked(dtype: str, count: int, fill) -> np.ndarray:
+    if dtype not in ("f32", "bf16"):
+        raise ValueError(f"unknown dtype {dtype!r}")
+    out = np.empty(count, dtype=np.float32 if dtype == "f32" else np.uint16)
+
+    def job(o):
+        n = min(_CHUNK, count - o)
+        out[o:o + n] = fill(o, n)
+
+    starts = range(0, count, _CHUNK)
+    if len(starts) <= 1:
+        for o in starts:
+            job(o)
+        return out
+    with cf.ThreadPoolExecutor(min(len(starts), os.cpu_count() or 1, 16)) as ex:
+        list(ex.map(job, starts))
+    return out
+
+
 def values(dtype: str, seed: int, stream: int, start: int, count: int,
            std: float = 1.0, mean: float = 0.0) -> np.ndarray:
     """``count`` consecutive values of one stream, stored in ``dtype``.
 
     Returns float32 for ``"f32"`` and uint16 bf16 bit patterns for ``"bf16"``.
     """
-    idx = np.arange(start, start + count, dtype=np.uint64)
-    v = normal_f32(seed, stream, idx, std, mean)
-    if dtype == "f32":
-        return v
-    if dtype == "bf16":
-        return f32_to_bf16_bits(v)
-    raise ValueError(f"unknown dtype {dtype!r}")
+    return _chunked(dtype, count, lambda o, n: _stored(
+        dtype, seed, stream, np.arange(start + o, start + o + n, dtype=np.uint64), std, mean))
 
 
 def values_at(dtype: str, seed: int, stream: int, index: np.ndarray,
               std: float = 1.0, mean: float = 0.0) -> np.ndarray:
     """Values of one stream at arbitrary flat indices (same as ``values``)."""
-    v = normal_f32(seed, stream, np.asarray(index, dtype=np.uint64), std, mean)
-    return v if dtype == "f32" else f32_to_bf16_bits(v)
+    index = np.asarray(index, dtype=np.uint64)
+    flat = index.reshape(-1)
+    out = _chunked(dtype, flat.size, lambda o, n: _stored(dtype, seed, stream, flat[o:o + n],
+                                                          std, mean))
+    return out.reshape(index.shape)
 
 
 def to_f64(dtype: str, stored: np.ndarray) -> np.ndarray:

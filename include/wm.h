@@ -189,6 +189,7 @@ wm_status wm_decode_attn(const wm_config* cfg, const wm_cache* cache, int32_t la
 
 /* Flags of wm_decode_attn_flags. */
 #define WM_ATTN_INPUTS_READY 1u
+#define WM_ATTN_DYNAMIC_SPLIT 2u
 
 /*
  * wm_decode_attn with flags; wm_decode_attn(...) is wm_decode_attn_flags(...,
@@ -204,6 +205,13 @@ wm_status wm_decode_attn(const wm_config* cfg, const wm_cache* cache, int32_t la
  *     layer's attention may share the workspace); it does NOT hold for the
  *     first layer after wm_kv_mix or after any update of seq_lens / the page
  *     table.
+ *   WM_ATTN_DYNAMIC_SPLIT: hand the KV stream out in chunks from a device
+ *     counter (about 8 chunks per warp, warps that stream faster take more)
+ *     whatever the launch size.  Without it only launches reading at least
+ *     2 GB of K/V do so; smaller ones give each warp one equal chunk.  The
+ *     result is the same within rounding (the merge order of the pieces of
+ *     a unit depends on where the chunks end, not on which warp takes them).
+ *     wm_decode_attn_workspace covers either split.
  * Unknown flag bits return WM_ERR_INVALID_ARG.
  */
 wm_status wm_decode_attn_flags(const wm_config* cfg, const wm_cache* cache, int32_t layer,
@@ -211,6 +219,17 @@ wm_status wm_decode_attn_flags(const wm_config* cfg, const wm_cache* cache, int3
                                const int32_t* seq_lens, int32_t B, int32_t max_pages, void* out,
                                void* workspace, size_t ws_bytes, uint32_t flags,
                                int32_t* dev_status, void* stream);
+
+/*
+ * How wm_decode_attn_flags would split a launch (no GPU work; for tuning and
+ * tests).  Fills plan[0..3] with: the persistent grid (CTAs), warps in it,
+ * work chunks it cuts the KV stream into at most, and stages (8 KB of K+V)
+ * per chunk, 0 meaning a static split with one chunk per warp.  The chunk
+ * count of a static split is its warp count.  Returns WM_ERR_INVALID_ARG for
+ * a bad config, B < 1, max_pages < 1, unknown flags or plan == NULL.
+ */
+wm_status wm_decode_attn_plan(const wm_config* cfg, int32_t B, int32_t max_pages, uint32_t flags,
+                              int32_t plan[4]);
 
 /*
  * Causal channel attention of one layer for many query positions at once:
@@ -268,8 +287,11 @@ wm_status wm_selftest_bounded_wait(int32_t* dev_status, uint32_t limit_us, void*
  *  - The first call on a device looks up that array's device address
  *    (cudaGetSymbolAddress) with the device current; make that first call
  *    before any stream capture.
- *  - Each call clears the part of the array that must start at zero (the
- *    arrival tickets) with an asynchronous memset on `stream`, then launches.
+ *  - Each call checks every argument first; only then does it clear the
+ *    span of the array its launch uses (arrival tickets and partial records,
+ *    so that nothing a call that timed out left behind counts as published)
+ *    with an asynchronous memset on `stream`, and launch.  A call refused on
+ *    the host writes nothing to the array.
  *  - All calls in the process share the one array per device: calls that
  *    overlap on the GPU (different streams without ordering) race and give
  *    wrong results.  Serialise them, e.g. on one stream.

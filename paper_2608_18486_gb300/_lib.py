@@ -18,8 +18,9 @@ WM_DT_F32, WM_DT_BF16 = 0, 1
 
 EXPORTED = ["wm_status_string", "wm_config_check", "wm_cache_bytes", "wm_cache_alloc",
             "wm_kv_mix_workspace", "wm_kv_mix", "wm_decode_attn_workspace", "wm_decode_attn",
-            "wm_decode_attn_flags", "wm_prefill_attn"]
+            "wm_decode_attn_flags", "wm_decode_attn_plan", "wm_prefill_attn"]
 WM_ATTN_INPUTS_READY = 1
+WM_ATTN_DYNAMIC_SPLIT = 2
 
 
 class wm_config(ctypes.Structure):
@@ -81,6 +82,9 @@ def lib():
         L.wm_decode_attn_flags.restype = ctypes.c_int
         L.wm_decode_attn_flags.argtypes = [cp, ctypes.POINTER(wm_cache), i32, vp, vp, vp, i32, i32,
                                            vp, vp, sz, ctypes.c_uint32, vp, vp]
+        L.wm_decode_attn_plan.restype = ctypes.c_int
+        L.wm_decode_attn_plan.argtypes = [cp, i32, i32, ctypes.c_uint32,
+                                          ctypes.POINTER(ctypes.c_int32)]
         L.wm_prefill_attn.restype = ctypes.c_int
         L.wm_prefill_attn.argtypes = [cp, ctypes.POINTER(wm_cache), i32, vp, vp, vp, i32, i32, i32,
                                       vp, vp, vp]
@@ -169,6 +173,15 @@ def wm_decode_attn_flags(cfg, cache, layer, q, page_table, seq_lens, B, max_page
                                       _p(page_table), _p(seq_lens), int(B), int(max_pages),
                                       _p(out), _p(workspace), int(ws_bytes), int(flags),
                                       _p(dev_status), stream)
+
+
+def wm_decode_attn_plan(cfg, B, max_pages, flags=0) -> dict:
+    """How a launch would be split: grid, warps, chunks, stages per chunk."""
+    plan = (ctypes.c_int32 * 4)()
+    rc = lib().wm_decode_attn_plan(ctypes.byref(cfg), int(B), int(max_pages), int(flags), plan)
+    if rc != WM_OK:
+        raise WMError(rc, "wm_decode_attn_plan")
+    return {"grid": plan[0], "warps": plan[1], "chunks": plan[2], "chunk_stages": plan[3]}
 
 
 def wm_prefill_attn(cfg, cache, layer, q, pos, page_table, B, Tq, max_pages, out, dev_status,

@@ -70,7 +70,7 @@ int64_t attn_chunk_capacity() {
          kAttnChunksPerWarp;
 }
 
-AttnPlan attn_plan(const wm_config& c, int32_t B, int32_t max_pages) {
+AttnPlan attn_plan(const wm_config& c, int32_t B, int32_t max_pages, bool force_dynamic = false) {
   AttnPlan pl{};
   const int64_t max_slots = (int64_t)max_pages * c.page_size;
   const double kv_bytes = (double)B * c.Hkv * max_slots * 2.0 * c.d * elem_size(c.dtype);
@@ -87,7 +87,7 @@ AttnPlan attn_plan(const wm_config& c, int32_t B, int32_t max_pages) {
   if (grid < 1) grid = 1;
   pl.grid = (int)grid;
   pl.nwarps = (int)grid * wpc;
-  if (kv_bytes >= kAttnDynamicLaunchBytes) {
+  if (force_dynamic || kv_bytes >= kAttnDynamicLaunchBytes) {
     int64_t ch = (ns_max + (int64_t)pl.nwarps * kAttnChunksPerWarp - 1) /
                  ((int64_t)pl.nwarps * kAttnChunksPerWarp);
     if (ch < kAttnMinChunkStages) ch = kAttnMinChunkStages;
@@ -129,6 +129,64 @@ wm_status check_cache(const wm_config& c, const wm_cache* cache) {
     return WM_ERR_INVALID_ARG;
   if (!aligned(cache->k_pool, 16) || !aligned(cache->v_pool, 16)) return WM_ERR_INVALID_ARG;
   return WM_OK;
+}
+
+// Checks, plans and launches one decode-attention call.  clear_workspace:
+// zero the span of the workspace the launch uses (counters and records) on
+// the stream just before the launch, after every argument check passed; the
+// fixed scratch of wm_decode_attn_noalloc keeps whatever the last call left.
+wm_status decode_attn_impl(const wm_config* c, const wm_cache* cache, int32_t layer, const void* q,
+                           const int32_t* page_table, const int32_t* seq_lens, int32_t B,
+                           int32_t max_pages, void* out, void* workspace, size_t ws_bytes,
+                           uint32_t flags, bool clear_workspace, int32_t* dev_status,
+                           void* stream) {
+  wm_status st = wm_config_check(c);
+  if (st != WM_OK) return st;
+  if (flags & ~(uint32_t)(WM_ATTN_INPUTS_READY | WM_ATTN_DYNAMIC_SPLIT)) return WM_ERR_INVALID_ARG;
+  if ((st = check_cache(*c, cache)) != WM_OK) return st;
+  if (layer < 0 || layer >= c->L || B < 0 || max_pages < 1) return WM_ERR_INVALID_ARG;
+  if ((int64_t)max_pages * c->page_size > INT32_MAX / 2) return WM_ERR_INVALID_ARG;
+  if (B == 0) return WM_OK;
+  if (B > kAttnMaxBatch) return WM_ERR_UNSUPPORTED;
+  if ((int64_t)B * c->Hq > INT32_MAX / 2) return WM_ERR_UNSUPPORTED;  // 32-bit output rows
+  if (!q || !page_table || !seq_lens || !out || !workspace) return WM_ERR_INVALID_ARG;
+  if (!aligned(q, 16) || !aligned(out, 16) || !aligned(workspace, 256)) return WM_ERR_INVALID_ARG;
+  const AttnPlan pl = attn_plan(*c, B, max_pages, (flags & WM_ATTN_DYNAMIC_SPLIT) != 0);
+  if (ws_bytes < pl.total) return WM_ERR_INVALID_ARG;
+  if (pl.max_chunks > attn_chunk_capacity()) return WM_ERR_UNSUPPORTED;  // cannot happen
+
+  const int chan = c->chan_of_layer[layer];
+  const size_t esz = elem_size(c->dtype);
+  const int64_t chan_elems = (int64_t)cache->num_pages * c->Hkv * c->page_size * c->d;
+  wm::AttnParams p{};
+  p.k_pool = (const char*)cache->k_pool + (size_t)chan * chan_elems * esz;
+  p.v_pool = (const char*)cache->v_pool + (size_t)chan * chan_elems * esz;
+  p.q = q;
+  p.out = out;
+  p.page_table = page_table;
+  p.seq_lens = seq_lens;
+  p.part = (float*)((char*)workspace + pl.off_part);
+  p.counters = (int32_t*)((char*)workspace + pl.off_counters);
+  p.status = dev_status;
+  p.page_stride = (int64_t)c->Hkv * c->page_size * c->d;
+  p.Hq = c->Hq;
+  p.Hkv = c->Hkv;
+  p.P = c->page_size;
+  p.log2P = ilog2(c->page_size);
+  p.num_pages = cache->num_pages;
+  p.max_pages = max_pages;
+  p.B = B;
+  p.chunk_stages = pl.chunk_stages;
+  p.max_chunks = pl.max_chunks;
+  p.inputs_ready = (flags & WM_ATTN_INPUTS_READY) ? 1 : 0;
+  p.epoch = next_attn_epoch();
+  p.qscale = (float)(1.4426950408889634 / sqrt((double)c->d));
+  if (clear_workspace &&
+      cudaMemsetAsync(workspace, 0, pl.total, (cudaStream_t)stream) != cudaSuccess)
+    return WM_ERR_CUDA;
+  cudaError_t e = wm::launch_decode_attn(p, pl.stage_bytes, c->dtype, c->d, c->Hq / c->Hkv,
+                                         pl.grid, (cudaStream_t)stream);
+  return e == cudaSuccess ? WM_OK : WM_ERR_CUDA;
 }
 
 }  // namespace
@@ -193,7 +251,22 @@ wm_status wm_cache_alloc(const wm_config* c, void* dev_buf, size_t bytes, int32_
 size_t wm_decode_attn_workspace(const wm_config* c, int32_t B, int32_t max_pages) {
   if (wm_config_check(c) != WM_OK || B < 0 || max_pages < 1) return 0;
   if (B == 0) return 256;
-  return attn_plan(*c, B, max_pages).total;
+  // enough for either split (WM_ATTN_DYNAMIC_SPLIT may cut more chunks)
+  const size_t a = attn_plan(*c, B, max_pages, false).total;
+  const size_t b = attn_plan(*c, B, max_pages, true).total;
+  return a > b ? a : b;
+}
+
+wm_status wm_decode_attn_plan(const wm_config* c, int32_t B, int32_t max_pages, uint32_t flags,
+                              int32_t plan[4]) {
+  if (wm_config_check(c) != WM_OK || B < 1 || max_pages < 1 || !plan) return WM_ERR_INVALID_ARG;
+  if (flags & ~(uint32_t)(WM_ATTN_INPUTS_READY | WM_ATTN_DYNAMIC_SPLIT)) return WM_ERR_INVALID_ARG;
+  const AttnPlan pl = attn_plan(*c, B, max_pages, (flags & WM_ATTN_DYNAMIC_SPLIT) != 0);
+  plan[0] = pl.grid;
+  plan[1] = pl.nwarps;
+  plan[2] = pl.max_chunks;
+  plan[3] = pl.chunk_stages;
+  return WM_OK;
 }
 
 wm_status wm_decode_attn(const wm_config* c, const wm_cache* cache, int32_t layer, const void* q,
@@ -208,51 +281,8 @@ wm_status wm_decode_attn_flags(const wm_config* c, const wm_cache* cache, int32_
                                const void* q, const int32_t* page_table, const int32_t* seq_lens,
                                int32_t B, int32_t max_pages, void* out, void* workspace,
                                size_t ws_bytes, uint32_t flags, int32_t* dev_status, void* stream) {
-  wm_status st = wm_config_check(c);
-  if (st != WM_OK) return st;
-  if (flags & ~(uint32_t)WM_ATTN_INPUTS_READY) return WM_ERR_INVALID_ARG;
-  if (st != WM_OK) return st;
-  if ((st = check_cache(*c, cache)) != WM_OK) return st;
-  if (layer < 0 || layer >= c->L || B < 0 || max_pages < 1) return WM_ERR_INVALID_ARG;
-  if ((int64_t)max_pages * c->page_size > INT32_MAX / 2) return WM_ERR_INVALID_ARG;
-  if (B == 0) return WM_OK;
-  if (B > kAttnMaxBatch) return WM_ERR_UNSUPPORTED;
-  if ((int64_t)B * c->Hq > INT32_MAX / 2) return WM_ERR_UNSUPPORTED;  // 32-bit output rows
-  if (!q || !page_table || !seq_lens || !out || !workspace) return WM_ERR_INVALID_ARG;
-  if (!aligned(q, 16) || !aligned(out, 16) || !aligned(workspace, 256)) return WM_ERR_INVALID_ARG;
-  const AttnPlan pl = attn_plan(*c, B, max_pages);
-  if (ws_bytes < pl.total) return WM_ERR_INVALID_ARG;
-  if (pl.max_chunks > attn_chunk_capacity()) return WM_ERR_UNSUPPORTED;  // cannot happen
-
-  const int chan = c->chan_of_layer[layer];
-  const size_t esz = elem_size(c->dtype);
-  const int64_t chan_elems = (int64_t)cache->num_pages * c->Hkv * c->page_size * c->d;
-  wm::AttnParams p{};
-  p.k_pool = (const char*)cache->k_pool + (size_t)chan * chan_elems * esz;
-  p.v_pool = (const char*)cache->v_pool + (size_t)chan * chan_elems * esz;
-  p.q = q;
-  p.out = out;
-  p.page_table = page_table;
-  p.seq_lens = seq_lens;
-  p.part = (float*)((char*)workspace + pl.off_part);
-  p.counters = (int32_t*)((char*)workspace + pl.off_counters);
-  p.status = dev_status;
-  p.page_stride = (int64_t)c->Hkv * c->page_size * c->d;
-  p.Hq = c->Hq;
-  p.Hkv = c->Hkv;
-  p.P = c->page_size;
-  p.log2P = ilog2(c->page_size);
-  p.num_pages = cache->num_pages;
-  p.max_pages = max_pages;
-  p.B = B;
-  p.chunk_stages = pl.chunk_stages;
-  p.max_chunks = pl.max_chunks;
-  p.inputs_ready = (flags & WM_ATTN_INPUTS_READY) ? 1 : 0;
-  p.epoch = next_attn_epoch();
-  p.qscale = (float)(1.4426950408889634 / sqrt((double)c->d));
-  cudaError_t e = wm::launch_decode_attn(p, pl.stage_bytes, c->dtype, c->d, c->Hq / c->Hkv,
-                                         pl.grid, (cudaStream_t)stream);
-  return e == cudaSuccess ? WM_OK : WM_ERR_CUDA;
+  return decode_attn_impl(c, cache, layer, q, page_table, seq_lens, B, max_pages, out, workspace,
+                          ws_bytes, flags, false, dev_status, stream);
 }
 
 wm_status wm_prefill_attn(const wm_config* c, const wm_cache* cache, int32_t layer,
@@ -440,10 +470,10 @@ extern "C" wm_status wm_decode_attn_noalloc(const wm_config* c, const wm_cache* 
   if (pl.total > (size_t)WM_NOALLOC_SCRATCH_BYTES) return WM_ERR_UNSUPPORTED;
   void* scratch = nullptr;
   if ((st = noalloc_scratch(&scratch)) != WM_OK) return st;
-  // the counters must start at zero; the array keeps the last call's bytes
-  if (cudaMemsetAsync((char*)scratch + pl.off_counters, 0, pl.off_part - pl.off_counters,
-                      (cudaStream_t)stream) != cudaSuccess)
-    return WM_ERR_CUDA;
-  return wm_decode_attn(c, cache, layer, q, page_table, seq_lens, B, max_pages, out, scratch,
-                        (size_t)WM_NOALLOC_SCRATCH_BYTES, dev_status, stream);
+  // The array keeps the last call's bytes.  Every argument is checked first;
+  // then the span this launch uses (arrival tickets, and the partial records
+  // whose flags a call that timed out may have left raised) is zeroed on the
+  // stream just before the launch.
+  return decode_attn_impl(c, cache, layer, q, page_table, seq_lens, B, max_pages, out, scratch,
+                          (size_t)WM_NOALLOC_SCRATCH_BYTES, 0u, true, dev_status, stream);
 }

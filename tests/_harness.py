@@ -48,83 +48,8 @@ def run_attn(sess, dp, layer) -> torch.Tensor:
 
 
 # ------------------------------------------------------------------ oracle side
-def oracle_attn_full(prob, layer, nthreads=8) -> np.ndarray:
-    w = prob.w
-    return O.decode_attn(prob.host("q")[layer], prob.host("k_pool"), prob.host("v_pool"),
-                         prob.page_table, prob.seq_lens, chan=prob.chan[layer], Hq=w.Hq,
-                         Hkv=w.Hkv, d=w.d, P=w.page, nthreads=nthreads)
-
-
-def oracle_attn_unit(prob, layer, b, hq) -> np.ndarray:
-    """One (sequence, query head) of one layer, from only that sequence's pages."""
-    w = prob.w
-    hkv = hq // (w.Hq // w.Hkv)
-    chan = prob.chan[layer]
-    S = int(prob.seq_lens[b])
-    npg = -(-S // w.page)
-    pages = prob.page_table[b, :npg].astype(np.int64)
-    s = np.arange(w.page, dtype=np.int64)
-    e = np.arange(w.d, dtype=np.int64)
-    # flat index of (chan, page, hkv, s, e) in the pool layout
-    base = ((chan * prob.num_pages + pages) * w.Hkv + hkv) * w.page
-    idx = ((base[:, None] + s[None, :]) * w.d)[:, :, None] + e[None, None, :]
-    kp = prob.at("k_pool", idx.reshape(-1)).reshape(1, npg, 1, w.page, w.d)
-    vp = prob.at("v_pool", idx.reshape(-1)).reshape(1, npg, 1, w.page, w.d)
-    qi = ((layer * w.B + b) * w.Hq + hq) * w.d + e
-    q = prob.at("q", qi).reshape(1, 1, w.d)
-    pt = np.arange(npg, dtype=np.int32).reshape(1, npg)
-    return O.decode_attn(q, kp, vp, pt, [S], chan=0, Hq=1, Hkv=1, d=w.d, P=w.page)[0, 0]
-
-
-def oracle_prefill_unit(prob, layer, b, pos, q_row) -> np.ndarray:
-    """Causal prefill attention of one query row (token position ``pos`` of
-    sequence b, query head given by ``q_row``'s head index), from only the
-    pages it reads.  ``q_row`` is (hq, d storage-dtype values)."""
-    w = prob.w
-    hq, qv = q_row
-    hkv = hq // (w.Hq // w.Hkv)
-    chan = prob.chan[layer]
-    npg = pos // w.page + 1
-    pages = prob.page_table[b, :npg].astype(np.int64)
-    s = np.arange(w.page, dtype=np.int64)
-    e = np.arange(w.d, dtype=np.int64)
-    base = ((chan * prob.num_pages + pages) * w.Hkv + hkv) * w.page
-    idx = ((base[:, None] + s[None, :]) * w.d)[:, :, None] + e[None, None, :]
-    kp = prob.at("k_pool", idx.reshape(-1)).reshape(1, npg, 1, w.page, w.d)
-    vp = prob.at("v_pool", idx.reshape(-1)).reshape(1, npg, 1, w.page, w.d)
-    pt = np.arange(npg, dtype=np.int32).reshape(1, npg)
-    q = np.ascontiguousarray(qv).reshape(1, 1, 1, w.d)
-    return O.prefill_attn(q, kp, vp, pt, np.array([[pos]], np.int32), chan=0, Hq=1, Hkv=1,
-                          d=w.d, P=w.page)[0, 0, 0]
-
-
-def oracle_mix_tokens(prob, tokens=None, chans=None):
-    """K~ and V of the chosen tokens and channels: dict[(b, j)] -> (K[Hkv][d], V[Hkv][d])."""
-    w = prob.w
-    tokens = range(w.B) if tokens is None else tokens
-    chans = range(w.k) if chans is None else chans
-    h = prob.host("h")
-    pre_g, br, ch_g, qk_g = (prob.host(n) for n in ("pre_g", "br", "ch_g", "qk_g"))
-    Wr = prob.host("Wr")
-    nout = w.Hkv * w.d
-    Wj = {}
-    for X in range(2):
-        for j in chans:
-            Wj[X, j] = prob.rows("Wkv", (X * w.k + j) * nout, nout, w.D)
-    res = {}
-    for b in tokens:
-        hhat, alpha, _ = O.pool_route(h[b], pre_g, Wr, br, L=w.L, k=w.k, D=w.D, p=w.p,
-                                      eps=w.eps_rms)
-        pos = float(prob.seq_lens[b]) - 1.0
-        for j in chans:
-            outs = []
-            for X in range(2):
-                _, o, _ = O.pool_channel(hhat[X], alpha[X, j], ch_g[X, j], Wj[X, j], qk_g[j],
-                                         is_key=(X == 0), pos=pos, Hkv=w.Hkv, d=w.d,
-                                         eps=w.eps_rms, eps_qk=w.eps_qk, theta=w.rope_theta)
-                outs.append(o.reshape(w.Hkv, w.d))
-            res[b, j] = tuple(outs)
-    return res
+from ._oracle_side import (oracle_attn_full, oracle_attn_layer, oracle_attn_unit,  # noqa: E402,F401
+                           oracle_mix_tokens, oracle_prefill_unit)
 
 
 def gpu_written_kv(sess, prob, b, j):

@@ -13,6 +13,21 @@ from wm_synth import configs
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
 
+def _cuda_present() -> bool:
+    try:
+        import torch
+        return torch.cuda.is_available()
+    except Exception:  # pragma: no cover
+        return False
+
+
+# Tests that hand made-up device addresses to entry points that can launch:
+# they check refusals made on the host before any launch, and run only where
+# no GPU could ever receive a launch should a check regress.
+host_refusals_only = pytest.mark.skipif(
+    _cuda_present(), reason="passes made-up device addresses; host-side checks only, CPU only")
+
+
 def declared_functions():
     names = set()
     for hdr in glob.glob(os.path.join(ROOT, "include", "*.h")):
@@ -69,6 +84,7 @@ def test_cache_sizing_and_layout_without_gpu():
     assert W.wm_cache_bytes(c, 0) == 0
 
 
+@host_refusals_only
 def test_compute_calls_reject_bad_arguments_before_launching():
     c = cfg()
     n = W.wm_cache_bytes(c, 4)
@@ -86,7 +102,7 @@ def test_compute_calls_reject_bad_arguments_before_launching():
     # a cache laid out for another config is refused
     other = cfg(k=8)
     assert W.wm_decode_attn(other, cache, 0, fake, fake, fake, 2, 4, fake, fake, ws, None, None) == W.WM_ERR_INVALID_ARG
-    assert W.wm_decode_attn_flags(c, cache, 0, fake, fake, fake, 2, 4, fake, fake, ws, 2, None,
+    assert W.wm_decode_attn_flags(c, cache, 0, fake, fake, fake, 2, 4, fake, fake, ws, 4, None,
                                   None) == W.WM_ERR_INVALID_ARG  # unknown flag bit
     wts = W.mix_weights((fake, fake), (fake, fake), (fake, fake), (fake, fake), (fake, fake), fake)
     mws = W.wm_kv_mix_workspace(c, 2)
@@ -96,6 +112,7 @@ def test_compute_calls_reject_bad_arguments_before_launching():
     assert W.wm_kv_mix(c, cache, wts, None, None, None, 0, 4, None, 0, None, None) == W.WM_OK
 
 
+@host_refusals_only
 def test_attention_refuses_output_rows_past_32_bits_before_launching():
     # 4096 sequences x 2^19 query heads: more output rows than the kernel's
     # 32-bit row index covers
@@ -122,6 +139,7 @@ def test_status_strings():
         assert W.wm_status_string(code) and W.wm_status_string(code) != "unknown status"
 
 
+@host_refusals_only
 def test_prefill_rejects_unsupported_and_bad_arguments_before_launching():
     c = cfg()
     n = W.wm_cache_bytes(c, 4)
@@ -146,3 +164,29 @@ def test_prefill_rejects_unsupported_and_bad_arguments_before_launching():
     # nothing to do is a no-op even with NULL buffers
     assert W.wm_prefill_attn(c, cache, 0, None, None, None, 0, 8, 4, None, None, None) == W.WM_OK
     assert W.wm_prefill_attn(c, cache, 0, None, None, None, 2, 0, 4, None, None, None) == W.WM_OK
+
+
+def test_attention_plan_static_and_dynamic_split():
+    # no_compression: 16 x 12 units of 2048 slots, 100 MB per launch -> static
+    w = configs.get("no_compression")
+    c = W.make_config(w.L, w.k, w.D, w.Hq, w.Hkv, w.d, w.p, w.page, w.dtype, w.chan_of_layer())
+    max_pages = -(-(w.ctx + 1) // w.page)
+    st = W.wm_decode_attn_plan(c, w.B, max_pages)
+    assert st["chunk_stages"] == 0 and st["chunks"] == st["warps"] > 0
+    dy = W.wm_decode_attn_plan(c, w.B, max_pages, W.WM_ATTN_DYNAMIC_SPLIT)
+    assert dy["grid"] == st["grid"] and dy["chunk_stages"] >= 4
+    assert dy["chunks"] > dy["warps"]  # warps take further chunks from the counter
+    # the workspace query covers either split
+    ws = W.wm_decode_attn_workspace(c, w.B, max_pages)
+    rec = 4 * (w.d + 4)  # one partial record at G = 1 (d outputs, m, l, flag; 16-byte padded)
+    assert ws >= 2 * dy["chunks"] * rec
+    # a launch of over 2 GB (the long-context workload) splits dynamically anyway
+    lw = configs.get("long128k")
+    lc = W.make_config(lw.L, lw.k, lw.D, lw.Hq, lw.Hkv, lw.d, lw.p, lw.page, lw.dtype,
+                       lw.chan_of_layer())
+    big = W.wm_decode_attn_plan(lc, lw.B, -(-(lw.ctx + 1) // lw.page))
+    assert big["chunk_stages"] > 0 and big["chunks"] > big["warps"]
+    with pytest.raises(W.WMError):
+        W.wm_decode_attn_plan(c, w.B, max_pages, 8)  # unknown flag bit
+    with pytest.raises(W.WMError):
+        W.wm_decode_attn_plan(c, 0, max_pages)

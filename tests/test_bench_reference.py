@@ -4,14 +4,17 @@ import json
 import os
 import subprocess
 import sys
+import time
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
 
 def test_reference_arm_prints_one_contract_line():
+    t0 = time.time()
     r = subprocess.run([sys.executable, "bench.py", "--impl", "reference", "--steps", "2",
                         "--warmup", "1", "--workload", "tiny_f32", "--ref-budget", "0.2"],
                        cwd=ROOT, capture_output=True, text=True, timeout=600)
+    wall = time.time() - t0
     assert r.returncode == 0, r.stderr[-2000:]
     lines = [l for l in r.stdout.splitlines() if l.startswith("{")]
     assert len(lines) == 1
@@ -24,3 +27,6 @@ def test_reference_arm_prints_one_contract_line():
     assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["sample"] and cb["value"] == d["value"]
     assert d["e2e"] == {"value": d["value"], "unit": "tokens/s", "h2d_bytes_per_step": 0,
                         "d2h_bytes_per_step": 0}
+    # the steps it reports are the steps it ran: their time fits in the run
+    assert d["steps"] * d["ms_per_step"] / 1e3 <= wall
+    assert d["extrapolated"]["ms_per_full_step"] > 0

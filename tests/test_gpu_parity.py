@@ -182,7 +182,7 @@ def _sample_units(w, prob, n, rng):
 
 @pytest.mark.parametrize("name,layers,nunits", [
     ("compress50", None, 6), ("large", (0, 13, 31), 3), ("long32k", (0, 31), 2),
-    ("long128k", (5,), 2)])
+    ("long64k", (7, 30), 2), ("long128k", (5,), 2)])
 def test_full_size_attention_sampled(name, layers, nunits):
     w = configs.get(name)
     prob, sess, dp = H.setup(w)

@@ -64,3 +64,31 @@ def test_chunked_generation_equals_the_one_pass_definition():
         ref = gen.normal_f32(5, 9, idx, 0.3, -0.2)
         assert at.shape == idx.shape
         assert np.array_equal(at, ref if dtype == "f32" else gen.f32_to_bf16_bits(ref))
+
+
+def test_compiled_host_generator_equals_the_numpy_definition():
+    """gen_host.c (the fast host fill) gives every bit the numpy definition
+    gives, for consecutive runs and scattered indices, both storage dtypes."""
+    L = gen._host_lib()
+    assert L is not None, "gen_host.c did not build"
+    rng = np.random.default_rng(7)
+    for dtype in ("f32", "bf16"):
+        for seed, stream, start, n, std, mean in [(0, 30, 0, 100003, 1.0, 0.0),
+                                                  (3, 4, 2 ** 33 + 5, 70001, 0.1, 1.0),
+                                                  (1, 40, 12345, 1, 8.0, 0.0),
+                                                  (2, 10, 2 ** 40, 300000, 0.0625, -0.5)]:
+            a = gen.values(dtype, seed, stream, start, n, std, mean)
+            b = gen.values_np(dtype, seed, stream, start, n, std, mean)
+            assert a.dtype == b.dtype and np.array_equal(a, b), (dtype, seed, stream)
+            idx = rng.integers(0, 2 ** 50, size=(3, 1001)).astype(np.uint64)
+            a = gen.values_at(dtype, seed, stream, idx, std, mean)
+            b = gen.values_at_np(dtype, seed, stream, idx, std, mean)
+            assert a.shape == idx.shape and np.array_equal(a, b)
+
+
+def test_runs_gather_equals_consecutive_values():
+    starts = np.array([5, 2 ** 35 + 3, 999, 5], dtype=np.uint64)
+    for dtype in ("f32", "bf16"):
+        got = gen.values_runs(dtype, 4, 31, starts, 4097, 0.5, 0.25)
+        for r, s0 in enumerate(starts):
+            assert np.array_equal(got[r], gen.values_np(dtype, 4, 31, int(s0), 4097, 0.5, 0.25))

@@ -2,7 +2,8 @@
 
 This module holds no arithmetic of the method; it only turns
 ``(seed, stream, flat index)`` into a synthetic value, identically on the host
-(numpy, here) and on the device (``synth.cu`` in this folder).
+(numpy here, and the same definition compiled in ``gen_host.c``) and on the
+device (``synth.cu`` in this folder).
 
 Definition
 ----------
@@ -23,7 +24,9 @@ Definition
 from __future__ import annotations
 
 import concurrent.futures as cf
+import ctypes
 import os
+import subprocess
 
 import numpy as np
 
@@ -120,9 +123,10 @@ def _chunked(dtype: str, count: int, fill) -> np.ndarray:
     return out
 
 
-def values(dtype: str, seed: int, stream: int, start: int, count: int,
-           std: float = 1.0, mean: float = 0.0) -> np.ndarray:
-    """``count`` consecutive values of one stream, stored in ``dtype``.
+def values_np(dtype: str, seed: int, stream: int, start: int, count: int,
+              std: float = 1.0, mean: float = 0.0) -> np.ndarray:
+    """``count`` consecutive values of one stream, stored in ``dtype``, computed
+    with numpy from the definition above.
 
     Returns float32 for ``"f32"`` and uint16 bf16 bit patterns for ``"bf16"``.
     """
@@ -130,14 +134,107 @@ def values(dtype: str, seed: int, stream: int, start: int, count: int,
         dtype, seed, stream, np.arange(start + o, start + o + n, dtype=np.uint64), std, mean))
 
 
-def values_at(dtype: str, seed: int, stream: int, index: np.ndarray,
-              std: float = 1.0, mean: float = 0.0) -> np.ndarray:
-    """Values of one stream at arbitrary flat indices (same as ``values``)."""
+def values_at_np(dtype: str, seed: int, stream: int, index: np.ndarray,
+                 std: float = 1.0, mean: float = 0.0) -> np.ndarray:
+    """Values of one stream at arbitrary flat indices (numpy, same as ``values_np``)."""
     index = np.asarray(index, dtype=np.uint64)
     flat = index.reshape(-1)
     out = _chunked(dtype, flat.size, lambda o, n: _stored(dtype, seed, stream, flat[o:o + n],
                                                           std, mean))
     return out.reshape(index.shape)
+
+
+# The same definition compiled (gen_host.c, OpenMP): tens of times faster than
+# numpy for the gigabyte-sized regenerations of the full-size parity tests.
+# Built on first use; without a C compiler the numpy functions serve.
+_HERE = os.path.dirname(os.path.abspath(__file__))
+HOST_SRC = os.path.join(_HERE, "gen_host.c")
+HOST_LIB = os.path.join(_HERE, "libwmgen.so")
+_host = None
+
+
+def build_host(verbose: bool = False) -> str:
+    cmd = ["gcc", "-O2", "-std=c11", "-fopenmp", "-ffp-contract=off", "-shared", "-fPIC",
+           "-o", HOST_LIB, HOST_SRC]
+    if verbose:
+        print(" ".join(cmd))
+    subprocess.check_call(cmd)
+    return HOST_LIB
+
+
+def _host_lib():
+    global _host
+    if _host is None:
+        try:
+            if not os.path.exists(HOST_LIB) or os.path.getmtime(HOST_LIB) < os.path.getmtime(HOST_SRC):
+                build_host()
+            L = ctypes.CDLL(HOST_LIB)
+            L.wmg_fill_runs.restype = None
+            L.wmg_fill_runs.argtypes = [ctypes.c_int, ctypes.c_uint64, ctypes.c_void_p,
+                                        ctypes.c_int64, ctypes.c_int64, ctypes.c_float,
+                                        ctypes.c_float, ctypes.c_float, ctypes.c_void_p,
+                                        ctypes.c_int]
+            L.wmg_fill.restype = None
+            L.wmg_fill.argtypes = [ctypes.c_int, ctypes.c_uint64, ctypes.c_uint64, ctypes.c_int64,
+                                   ctypes.c_void_p, ctypes.c_float, ctypes.c_float, ctypes.c_float,
+                                   ctypes.c_void_p, ctypes.c_int]
+            _host = L
+        except Exception:
+            _host = False
+    return _host or None
+
+
+def _fill_host(L, dtype, seed, stream, start, count, index, std, mean):
+    if dtype not in ("f32", "bf16"):
+        raise ValueError(f"unknown dtype {dtype!r}")
+    out = np.empty(count, dtype=np.float32 if dtype == "f32" else np.uint16)
+    key = int(stream_key(seed, stream))
+    L.wmg_fill(0 if dtype == "f32" else 1, key, int(start), int(count),
+               None if index is None else index.ctypes.data, float(IRWIN_HALL4_SCALE),
+               float(np.float32(std)), float(np.float32(mean)), out.ctypes.data, 0)
+    return out
+
+
+def values(dtype: str, seed: int, stream: int, start: int, count: int,
+           std: float = 1.0, mean: float = 0.0) -> np.ndarray:
+    """``count`` consecutive values of one stream, stored in ``dtype``.
+
+    Returns float32 for ``"f32"`` and uint16 bf16 bit patterns for ``"bf16"``.
+    """
+    L = _host_lib()
+    if L is None:
+        return values_np(dtype, seed, stream, start, count, std, mean)
+    return _fill_host(L, dtype, seed, stream, start, count, None, std, mean)
+
+
+def values_at(dtype: str, seed: int, stream: int, index: np.ndarray,
+              std: float = 1.0, mean: float = 0.0) -> np.ndarray:
+    """Values of one stream at arbitrary flat indices (same as ``values``)."""
+    L = _host_lib()
+    if L is None:
+        return values_at_np(dtype, seed, stream, index, std, mean)
+    index = np.ascontiguousarray(index, dtype=np.uint64)
+    out = _fill_host(L, dtype, seed, stream, 0, index.size, index.reshape(-1), std, mean)
+    return out.reshape(index.shape)
+
+
+def values_runs(dtype: str, seed: int, stream: int, starts, run_len: int,
+                std: float = 1.0, mean: float = 0.0) -> np.ndarray:
+    """[len(starts)][run_len] values: row r holds the run of ``run_len``
+    consecutive values from flat index ``starts[r]`` (same as ``values``)."""
+    starts = np.ascontiguousarray(starts, dtype=np.uint64).reshape(-1)
+    L = _host_lib()
+    if L is None:
+        return np.stack([values_np(dtype, seed, stream, int(s0), run_len, std, mean)
+                         for s0 in starts]) if len(starts) else \
+            np.empty((0, run_len), np.float32 if dtype == "f32" else np.uint16)
+    if dtype not in ("f32", "bf16"):
+        raise ValueError(f"unknown dtype {dtype!r}")
+    out = np.empty((starts.size, run_len), dtype=np.float32 if dtype == "f32" else np.uint16)
+    L.wmg_fill_runs(0 if dtype == "f32" else 1, int(stream_key(seed, stream)), starts.ctypes.data,
+                    starts.size, int(run_len), float(IRWIN_HALL4_SCALE), float(np.float32(std)),
+                    float(np.float32(mean)), out.ctypes.data, 0)
+    return out
 
 
 def to_f64(dtype: str, stored: np.ndarray) -> np.ndarray:

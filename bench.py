@@ -500,16 +500,17 @@ def run_gpu(args, w):
 
 def run_model(args, w):
     """Whole-model decode step: random Qwen3-style blocks (Sec. 4.1) around the
-    WhiteMatter path.  Per layer l: x = RMSNorm(h); q = RoPE(QKNorm(W_q x));
-    h += W_o * attention over channel c(l) (wm_decode_attn); h += SwiGLU MLP of
-    RMSNorm(h).  The L states entering the layers then go through the pool
-    (wm_kv_mix), as in Sec. 3.2.  The blocks are plain torch (cuBLAS GEMMs):
-    they are outside the path and only give the path its real neighbours.
-    Prints one JSON line: whole-model tokens/s and the WhiteMatter share."""
+    WhiteMatter path (tests/_model_step.py).  Per layer l: x = RMSNorm(h);
+    q = RoPE(QKNorm(W_q x)); h += W_o * attention over channel c(l)
+    (wm_decode_attn); h += SwiGLU MLP of RMSNorm(h).  The L states entering
+    the layers then go through the pool (wm_kv_mix), as in Sec. 3.2.  The
+    blocks are plain torch (cuBLAS GEMMs): they are outside the path and only
+    give the path its real neighbours.  Prints one JSON line: whole-model
+    tokens/s and the WhiteMatter share."""
     import torch
-    import torch.nn.functional as F
     from paper_2608_18486_gb300 import make_config
     from paper_2608_18486_gb300.session import DecodeSession
+    from tests._model_step import ModelStep
     from wm_synth.device_problem import DeviceProblem
 
     dev = torch.device("cuda", 0)
@@ -520,62 +521,12 @@ def run_model(args, w):
     sess = DecodeSession(cfg, w.B, prob.num_pages, prob.max_pages, dev)
     dp = DeviceProblem(prob, sess.k_pool, sess.v_pool, dev)
     sess.set_weights(*dp.weights())
-    dt = sess.dtype
-    I = args.intermediate or 3 * w.D
-    g = torch.Generator(device=dev).manual_seed(1)
-
-    def rnd(*shape, std):
-        return (torch.randn(*shape, generator=g, device=dev) * std).to(dt)
-
-    Wq = rnd(w.L, w.Hq * w.d, w.D, std=w.D ** -0.5)
-    Wo = rnd(w.L, w.D, w.Hq * w.d, std=(w.Hq * w.d) ** -0.5)
-    Wg = rnd(w.L, I, w.D, std=w.D ** -0.5)
-    Wu = rnd(w.L, I, w.D, std=w.D ** -0.5)
-    Wd = rnd(w.L, w.D, I, std=I ** -0.5)
-    # rotary angles of each sequence's new token (position seq_len - 1)
-    pos = dp.seq_lens.to(torch.float64) - 1.0
-    inv = w.rope_theta ** (-torch.arange(0, w.d // 2, device=dev, dtype=torch.float64) * 2.0 / w.d)
-    ang = pos[:, None] * inv[None, :]
-    cos = torch.cos(ang).float()[:, None, :]
-    sin = torch.sin(ang).float()[:, None, :]
-    h0 = rnd(w.B, w.D, std=1.0)
-    H = torch.empty((w.B, w.L, w.D), dtype=dt, device=dev)
-    q = torch.empty((w.L, w.B, w.Hq, w.d), dtype=dt, device=dev)
-    out = torch.empty((w.L, w.B, w.Hq, w.d), dtype=dt, device=dev)
+    model = ModelStep(w, sess, dp, dev, args.intermediate)
     stream = torch.cuda.Stream(dev)
-
-    def rms(x, eps):
-        xf = x.float()
-        return xf * torch.rsqrt(xf.pow(2).mean(-1, keepdim=True) + eps)
-
-    def model_step(ev=None):
-        h = h0
-        for l in range(w.L):
-            H[:, l] = h
-            x = rms(h, w.eps_rms).to(dt)
-            ql = rms((x @ Wq[l].T).view(w.B, w.Hq, w.d), w.eps_qk)
-            q1, q2 = ql[..., : w.d // 2], ql[..., w.d // 2:]
-            q[l] = torch.cat([q1 * cos - q2 * sin, q2 * cos + q1 * sin], -1).to(dt)
-            if ev is not None:
-                ev[l][0].record(stream)
-            # layer 0 follows the previous step's pool, which wrote the cache
-            sess.decode_attn(l, q[l], dp.page_table, dp.seq_lens, out[l], stream=stream,
-                             inputs_ready=l > 0)
-            if ev is not None:
-                ev[l][1].record(stream)
-            h = h + out[l].view(w.B, -1) @ Wo[l].T
-            x2 = rms(h, w.eps_rms).to(dt)
-            h = h + (F.silu(x2 @ Wg[l].T) * (x2 @ Wu[l].T)) @ Wd[l].T
-        if ev is not None:
-            ev[w.L][0].record(stream)
-        sess.kv_mix(H, dp.page_table, dp.slot, stream=stream)
-        if ev is not None:
-            ev[w.L][1].record(stream)
-        return h
 
     with torch.cuda.stream(stream):
         for _ in range(args.warmup):
-            model_step()
+            model.step(stream)
     torch.cuda.synchronize()
     K = args.steps
     evs = [[(torch.cuda.Event(enable_timing=True, external=True),
@@ -584,7 +535,7 @@ def run_model(args, w):
     graph = torch.cuda.CUDAGraph()
     with torch.cuda.graph(graph, stream=stream):
         for i in range(K):
-            model_step(evs[i])
+            model.step(stream, evs[i])
     with torch.cuda.stream(stream):
         graph.replay()
     torch.cuda.synchronize()
@@ -603,7 +554,7 @@ def run_model(args, w):
             "value": w.B * K / (ms / 1e3), "unit": "tokens/s", "n_gpus": 1, "steps": K,
             "warmup": args.warmup, "ms_per_step": ms / K, "higher_is_better": True,
             "dtype": w.dtype, "data": "synthetic",
-            "config": dict(config_dict(w, 1), intermediate=I, mode="model"),
+            "config": dict(config_dict(w, 1), intermediate=model.I, mode="model"),
             "whitematter_share": (attn_ms + mix_ms) / ms,
             "attn_ms_per_step": attn_ms / K, "pool_ms_per_step": mix_ms / K}
     print(json.dumps(line), flush=True)

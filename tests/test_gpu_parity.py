@@ -23,10 +23,14 @@ def _free():
 
 
 # ------------------------------------------------------------ small, complete
-@pytest.mark.parametrize("name", ["tiny_f32", "no_compression"])
-def test_attention_all_layers_all_heads(name):
-    w = configs.get(name)
-    prob, sess, dp = H.setup(w)
+@pytest.mark.parametrize("name,seed,q_scale", [
+    ("tiny_f32", 0, 1.0), ("no_compression", 0, 1.0), ("no_compression", 1, 1.0),
+    ("no_compression", 0, 8.0), ("no_compression", 1, 8.0)])
+def test_attention_all_layers_all_heads(name, seed, q_scale):
+    """q_scale 8: peaked attention (a few slots carry most of the weight),
+    where bf16 rounding of the softmax inputs matters most."""
+    w = configs.get(name).with_(q_scale=q_scale)
+    prob, sess, dp = H.setup(w, seed=seed)
     for layer in range(w.L):
         got = H.to_f64(H.run_attn(sess, dp, layer))
         want = H.oracle_attn_full(prob, layer)
@@ -35,10 +39,11 @@ def test_attention_all_layers_all_heads(name):
     _free()
 
 
-@pytest.mark.parametrize("name", ["tiny_f32", "no_compression"])
-def test_kv_mix_all_tokens_all_channels(name):
+@pytest.mark.parametrize("name,seed", [("tiny_f32", 0), ("no_compression", 0),
+                                       ("no_compression", 1)])
+def test_kv_mix_all_tokens_all_channels(name, seed):
     w = configs.get(name)
-    prob, sess, dp = H.setup(w)
+    prob, sess, dp = H.setup(w, seed=seed)
     sess.kv_mix(dp.h, dp.page_table, dp.slot)
     torch.cuda.synchronize()
     assert sess.read_status() == 0

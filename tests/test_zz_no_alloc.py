@@ -57,6 +57,31 @@ def test_noalloc_matches_workspace_entry_point_on_two_calls(name, overrides):
 NOALLOC_SCRATCH_BYTES = 8 << 20
 
 
+def test_noalloc_near_its_scratch_limit_on_two_calls():
+    """A launch whose partial records fill most of the fixed array (24
+    sequences, 16 query heads over 2 kv heads of 96: about 7.7 MB of records
+    over a full grid) gives the workspace entry point's rows on two calls in
+    a row: the record offsets and the cleared span reach the array's end."""
+    w = configs.get("paper_k16").with_(B=24, L=2, k=2, Hq=16, Hkv=2)
+    prob, sess, dp = H.setup(w)
+    plan = W.wm_decode_attn_plan(sess.cfg, w.B, prob.max_pages)
+    rec_bytes = 4 * (8 * 96 + 20)  # G = 8 heads of 96, (m, l) pairs and the flag, padded
+    used = 2 * plan["chunks"] * rec_bytes
+    assert plan["chunk_stages"] == 0 and 6 * 2 ** 20 < used < NOALLOC_SCRATCH_BYTES - 64 * 1024, plan
+    for layer in range(w.L):
+        ref = H.run_attn(sess, dp, layer)
+        outs = []
+        for _ in range(2):
+            out = torch.full_like(ref, float("nan"))
+            assert _noalloc(sess, dp, layer, out) == W.WM_OK
+            outs.append(out)
+        torch.cuda.synchronize()
+        assert sess.read_status() == 0
+        for out in outs:
+            err = H.rel_err(H.to_f64(out), H.to_f64(ref))
+            assert err <= H.TOL[w.dtype], (layer, err)
+
+
 def test_noalloc_rejects_launches_larger_than_its_scratch():
     # 4096 sequences x 8 query heads per kv head over 2 pages each: the
     # partial records alone need far more than the fixed array

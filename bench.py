@@ -325,6 +325,7 @@ def run_gpu(args, w):
     if world > 1 and not dist.is_initialized():
         dist.init_process_group("nccl", device_id=dev)
 
+    from paper_2608_18486_gb300 import _lib as W
     from paper_2608_18486_gb300 import make_config
     from paper_2608_18486_gb300.session import DecodeSession
     from wm_synth import configs as C
@@ -490,7 +491,7 @@ def run_gpu(args, w):
                                               + dp.h.numel() * dp.h.element_size()),
                     "d2h_bytes_per_step": int(outs.numel() * outs.element_size())},
             "clocks": clocks,
-            "gpu_launches": args.steps * (w.L + 5),
+            "gpu_launches": args.steps * (w.L + W.wm_kv_mix_launches(cfg, w.B)),
         }
         print(json.dumps(line), flush=True)
     if world > 1:
@@ -656,6 +657,11 @@ def run_prefill(args, w):
     print(json.dumps(line), flush=True)
 
 
+def sess_launches(sess, B):
+    from paper_2608_18486_gb300 import _lib as W
+    return W.wm_kv_mix_launches(sess.cfg, B)
+
+
 def run_pool(args, w):
     """The cross-layer KV pool (Sec. 3.1 Steps 1-2) over the B tokens of one
     batched evaluation: a prefill group of Sec. 3.3 hands the pool |G_q| x
@@ -723,7 +729,7 @@ def run_pool(args, w):
             "roofline": {"bound": "tensor", "achieved": tflops, "peak": peak, "unit": "TFLOP/s",
                          "frac": tflops / peak, "peak_kind": "measured sustained bf16",
                          "flops_per_step": flops, "bytes_per_step": wcfg.mix_bytes(w)},
-            "clocks": clocks, "gpu_launches": K * 4}
+            "clocks": clocks, "gpu_launches": K * sess_launches(sess, w.B)}
     t_cpu, cores, sample = oracle_pool_estimate(prob, budget_s=args.ref_budget)
     line["cpu_baseline"] = {"value": w.B / t_cpu, "unit": "tokens/s", "cores": cores,
                             "kind": "oracle", "sample": sample}

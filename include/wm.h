@@ -149,6 +149,8 @@ size_t wm_kv_mix_workspace(const wm_config* cfg, int32_t B);
  *   slot       device int32 [B]: write slot, 1 <= slot[b] < max_pages*page_size
  *   workspace  device, >= wm_kv_mix_workspace(cfg, B) bytes, 256-byte aligned,
  *              no contents required
+ * h, Wr, Wkv, pre_g and ch_g must be 16-byte aligned (WM_ERR_INVALID_ARG
+ * otherwise): they are read as 16-byte vectors.
  * Only the B*k*2*Hkv*d cache elements addressed are written.  A bad slot or
  * page id skips that token's write and sets WM_ERR_BOUNDS.  B = 0 is a no-op.
  */
@@ -156,6 +158,12 @@ wm_status wm_kv_mix(const wm_config* cfg, const wm_cache* cache, const wm_mix_we
                     const void* h, const int32_t* page_table, const int32_t* slot, int32_t B,
                     int32_t max_pages, void* workspace, size_t ws_bytes, int32_t* dev_status,
                     void* stream);
+
+/* Kernels one wm_kv_mix call of B tokens enqueues (0 for B = 0), -1 for an
+ * invalid config or B < 0; no GPU work: prenorm, router, mix and the
+ * projection with its fused epilogue (4 for bf16), or a separate epilogue
+ * after a SIMT projection (5: fp32, or no TMA encoder in the driver). */
+int32_t wm_kv_mix_launches(const wm_config* cfg, int32_t B);
 
 /* Workspace bytes wm_decode_attn needs for B sequences whose page tables
  * have max_pages entries. */

@@ -18,7 +18,8 @@ WM_DT_F32, WM_DT_BF16 = 0, 1
 
 EXPORTED = ["wm_status_string", "wm_config_check", "wm_cache_bytes", "wm_cache_alloc",
             "wm_kv_mix_workspace", "wm_kv_mix", "wm_decode_attn_workspace", "wm_decode_attn",
-            "wm_decode_attn_flags", "wm_decode_attn_plan", "wm_prefill_attn"]
+            "wm_decode_attn_flags", "wm_decode_attn_plan", "wm_prefill_attn",
+            "wm_kv_mix_launches"]
 WM_ATTN_INPUTS_READY = 1
 WM_ATTN_DYNAMIC_SPLIT = 2
 
@@ -82,6 +83,8 @@ def lib():
         L.wm_decode_attn_flags.restype = ctypes.c_int
         L.wm_decode_attn_flags.argtypes = [cp, ctypes.POINTER(wm_cache), i32, vp, vp, vp, i32, i32,
                                            vp, vp, sz, ctypes.c_uint32, vp, vp]
+        L.wm_kv_mix_launches.restype = ctypes.c_int32
+        L.wm_kv_mix_launches.argtypes = [cp, i32]
         L.wm_decode_attn_plan.restype = ctypes.c_int
         L.wm_decode_attn_plan.argtypes = [cp, i32, i32, ctypes.c_uint32,
                                           ctypes.POINTER(ctypes.c_int32)]
@@ -173,6 +176,11 @@ def wm_decode_attn_flags(cfg, cache, layer, q, page_table, seq_lens, B, max_page
                                       _p(page_table), _p(seq_lens), int(B), int(max_pages),
                                       _p(out), _p(workspace), int(ws_bytes), int(flags),
                                       _p(dev_status), stream)
+
+
+def wm_kv_mix_launches(cfg, B) -> int:
+    """Kernels one wm_kv_mix call of B tokens enqueues (-1: invalid)."""
+    return int(lib().wm_kv_mix_launches(ctypes.byref(cfg), int(B)))
 
 
 def wm_decode_attn_plan(cfg, B, max_pages, flags=0) -> dict:

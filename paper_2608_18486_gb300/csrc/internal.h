@@ -112,6 +112,7 @@ struct MixWorkspace {
 
 MixWorkspace mix_workspace_layout(const wm_config& cfg, int32_t B, int sm_count);
 cudaError_t launch_kv_mix(MixParams& p, int dtype, cudaStream_t s);
+int kv_mix_launches(const MixParams& p, int dtype);  // kernels launch_kv_mix enqueues
 
 // tcgen05 projection with the fused key/value epilogue, and the tcgen05
 // router with split-K fp32 partials (bf16 only)

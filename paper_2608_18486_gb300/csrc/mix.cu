@@ -733,6 +733,13 @@ MixWorkspace mix_workspace_layout(const wm_config& cfg, int32_t B, int sm_count)
   return w;
 }
 
+int kv_mix_launches(const MixParams& p, int dtype) {
+  if (p.B == 0) return 0;
+  // prenorm, router, mix, then the tensor-core projection with its epilogue
+  // or a SIMT projection and a separate epilogue
+  return dtype == WM_DT_BF16 && proj_tc_supported(p) ? 4 : 5;
+}
+
 cudaError_t launch_kv_mix(MixParams& p, int dtype, cudaStream_t s) {
   if (dtype == WM_DT_F32) return launch_all<float>(p, s);
   return launch_all<__nv_bfloat16>(p, s);

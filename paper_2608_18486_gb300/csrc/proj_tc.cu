@@ -23,6 +23,7 @@
 #include <math.h>
 
 #include "internal.h"
+#include "kv_epi.cuh"
 #include "tc.cuh"
 
 namespace wm {
@@ -192,91 +193,20 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     }
     return;
   }
-  // per (token, head) epilogue: keys QK-norm + RoPE, bf16 write to the cache slot.
-  // Lane t handles the RoPE pairs (i, i + HD/2) for i = t, t + 32, ...
-  constexpr int HALF = HD / 2;
-  constexpr int NP = (HALF + 31) / 32;  // pairs per lane
-  const bool reporter = (mt == 0 && j == 0 && X == 0);
-  __nv_bfloat16* pool = X == 0 ? p.k_pool : p.v_pool;
-  float qg0[NP], qg1[NP];  // QK-norm gain of channel j, the same for every item of this CTA
-#pragma unroll
-  for (int t = 0; t < NP; ++t) {
-    const int i = lane + 32 * t;
-    qg0[t] = i < HALF ? __bfloat162float(p.qk_g[(int64_t)j * HD + i]) : 0.f;
-    qg1[t] = i < HALF ? __bfloat162float(p.qk_g[(int64_t)j * HD + i + HALF]) : 0.f;
-  }
-  const float* cs_tab = p.rope_smem_off > 0 ? rope_s : p.rope_cs;
-  // Each warp takes IPW items per round, their loads, reductions and stores
-  // interleaved so that the latencies overlap.
-  constexpr int IPW = 4;
-  constexpr int NW = kTcThreads / 32;
-  const int nitems = nb * HPT;
-  for (int it0 = warp * IPW; it0 < nitems; it0 += NW * IPW) {
-    float y0[IPW][NP], y1[IPW][NP];
-    int n_[IPW], hh_[IPW], pg_[IPW];
-    bool on[IPW];
-#pragma unroll
-    for (int q = 0; q < IPW; ++q) {
-      const int it = it0 + q;
-      const int n = it / HPT, hl = it % HPT;  // n: token within the tile
-      n_[q] = n;
-      hh_[q] = mt * HPT + hl;
-      pg_[q] = it < nitems ? s_page[n] : -1;
-      on[q] = it < nitems && hh_[q] < p.Hkv && pg_[q] >= 0;
-      if (it < nitems && hh_[q] < p.Hkv && pg_[q] < 0 && reporter && hl == 0 && lane == 0)
-        report(p.status, WM_ERR_BOUNDS);
-      const float* src = T + n * kTcM + hl * HD;
-#pragma unroll
-      for (int t = 0; t < NP; ++t) {
-        const int i = lane + 32 * t;
-        y0[q][t] = on[q] && i < HALF ? src[i] : 0.f;
-        y1[q][t] = on[q] && i < HALF ? src[i + HALF] : 0.f;
-      }
-    }
-    if (X == 0) {
-      float ss[IPW];
-#pragma unroll
-      for (int q = 0; q < IPW; ++q) {
-        ss[q] = 0.f;
-#pragma unroll
-        for (int t = 0; t < NP; ++t) ss[q] = fmaf(y0[q][t], y0[q][t], fmaf(y1[q][t], y1[q][t], ss[q]));
-      }
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1)
-#pragma unroll
-        for (int q = 0; q < IPW; ++q) ss[q] += __shfl_xor_sync(0xFFFFFFFFu, ss[q], o);
-#pragma unroll
-      for (int q = 0; q < IPW; ++q) {
-        const float rr = rsqrtf(ss[q] / (float)HD + p.eps_qk);
-        const int row = cs_tab == rope_s ? n_[q] : n0 + n_[q];
-#pragma unroll
-        for (int t = 0; t < NP; ++t) {
-          const int i = lane + 32 * t;
-          if (on[q] && i < HALF) {
-            const float x0 = y0[q][t] * rr * qg0[t], x1 = y1[q][t] * rr * qg1[t];
-            const float2 csn = reinterpret_cast<const float2*>(cs_tab)[row * HALF + i];
-            y0[q][t] = x0 * csn.x - x1 * csn.y;  // rotate-half RoPE
-            y1[q][t] = x1 * csn.x + x0 * csn.y;
-          }
-        }
-      }
-    }
-#pragma unroll
-    for (int q = 0; q < IPW; ++q) {
-      if (!on[q]) continue;
-      const int s = s_slot[n_[q]];
-      __nv_bfloat16* dst =
-          pool + ((((int64_t)j * p.num_pages + pg_[q]) * p.Hkv + hh_[q]) * p.P + (s & (p.P - 1))) * HD;
-#pragma unroll
-      for (int t = 0; t < NP; ++t) {
-        const int i = lane + 32 * t;
-        if (i < HALF) {
-          dst[i] = __float2bfloat16_rn(y0[q][t]);
-          dst[i + HALF] = __float2bfloat16_rn(y1[q][t]);
-        }
-      }
-    }
-  }
+  // per (token, head) epilogue: keys QK-norm + RoPE, bf16 write to the cache slot
+  KvEpiArgs ea;
+  ea.Hkv = p.Hkv;
+  ea.P = p.P;
+  ea.num_pages = p.num_pages;
+  ea.eps_qk = p.eps_qk;
+  ea.qk_g = p.qk_g;
+  ea.k_pool = p.k_pool;
+  ea.v_pool = p.v_pool;
+  ea.status = p.status;
+  const bool local_tab = p.rope_smem_off > 0;
+  kv_epilogue_tile<HD, kTcThreads / 32>(T, nb, mt, j, X, nullptr, s_slot, s_page,
+                                        local_tab ? rope_s : p.rope_cs, local_tab ? 0 : n0,
+                                        mt == 0 && j == 0 && X == 0, ea);
 }
 
 // Row-major bf16 matrix [rows][cols] as a 2-D tensor map with a 64 x box_rows box.

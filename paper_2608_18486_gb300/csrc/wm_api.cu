@@ -111,6 +111,22 @@ AttnPlan attn_plan(const wm_config& c, int32_t B, int32_t max_pages, bool force_
   return pl;
 }
 
+// Shape fields of the pool's launch parameters.
+void mix_shape(const wm_config& c, int32_t B, wm::MixParams& p) {
+  p.B = B;
+  p.L = c.L;
+  p.k = c.k;
+  p.D = c.D;
+  p.Hkv = c.Hkv;
+  p.d = c.d;
+  p.p = c.p;
+  p.Lp = (c.L + c.p - 1) / c.p;
+  p.P = c.page_size;
+  p.log2P = ilog2(c.page_size);
+  p.eps_rms = c.eps_rms;
+  p.eps_qk = c.eps_qk;
+}
+
 // Tag of one attention call (never 0): a partial record counts as published
 // only when its flag holds the tag of the call reading it.
 int32_t next_attn_epoch() {
@@ -332,6 +348,15 @@ size_t wm_kv_mix_workspace(const wm_config* c, int32_t B) {
   return wm::mix_workspace_layout(*c, B, sm_count()).total;
 }
 
+int32_t wm_kv_mix_launches(const wm_config* c, int32_t B) {
+  if (wm_config_check(c) != WM_OK || B < 0) return -1;
+  wm::MixParams p{};
+  mix_shape(*c, B, p);
+  p.num_pages = 1;
+  p.max_pages = 1;
+  return wm::kv_mix_launches(p, c->dtype);
+}
+
 wm_status wm_kv_mix(const wm_config* c, const wm_cache* cache, const wm_mix_weights* w,
                     const void* h, const int32_t* page_table, const int32_t* slot, int32_t B,
                     int32_t max_pages, void* workspace, size_t ws_bytes, int32_t* dev_status,
@@ -348,26 +373,18 @@ wm_status wm_kv_mix(const wm_config* c, const wm_cache* cache, const wm_mix_weig
     if (!w->pre_g[X] || !w->Wr[X] || !w->br[X] || !w->ch_g[X] || !w->Wkv[X])
       return WM_ERR_INVALID_ARG;
   for (int X = 0; X < 2; ++X)
-    if (!aligned(w->Wr[X], 16) || !aligned(w->Wkv[X], 16)) return WM_ERR_INVALID_ARG;
+    if (!aligned(w->Wr[X], 16) || !aligned(w->Wkv[X], 16) || !aligned(w->pre_g[X], 16) ||
+        !aligned(w->ch_g[X], 16))
+      return WM_ERR_INVALID_ARG;
+  if (!aligned(h, 16)) return WM_ERR_INVALID_ARG;
   if (!aligned(workspace, 256)) return WM_ERR_INVALID_ARG;
   const wm::MixWorkspace ws = wm::mix_workspace_layout(*c, B, sm_count());
   if (ws_bytes < ws.total) return WM_ERR_INVALID_ARG;
 
   wm::MixParams p{};
-  p.B = B;
-  p.L = c->L;
-  p.k = c->k;
-  p.D = c->D;
-  p.Hkv = c->Hkv;
-  p.d = c->d;
-  p.p = c->p;
-  p.Lp = (c->L + c->p - 1) / c->p;
-  p.P = c->page_size;
-  p.log2P = ilog2(c->page_size);
+  mix_shape(*c, B, p);
   p.num_pages = cache->num_pages;
   p.max_pages = max_pages;
-  p.eps_rms = c->eps_rms;
-  p.eps_qk = c->eps_qk;
   p.h = h;
   for (int X = 0; X < 2; ++X) {
     p.pre_g[X] = w->pre_g[X];

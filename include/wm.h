@@ -153,6 +153,12 @@ size_t wm_kv_mix_workspace(const wm_config* cfg, int32_t B);
  * otherwise): they are read as 16-byte vectors.
  * Only the B*k*2*Hkv*d cache elements addressed are written.  A bad slot or
  * page id skips that token's write and sets WM_ERR_BOUNDS.  B = 0 is a no-op.
+ * The kernels are chained with programmatic dependent launch; the router and
+ * projection kernels start streaming their weights (Wr, Wkv) before waiting
+ * for the work before them, which is the library's own previous kernel.  So
+ * the weights must not be written by a kernel that runs immediately before
+ * the call and lets its dependents start early (ordinary kernels and copies
+ * do not).
  */
 wm_status wm_kv_mix(const wm_config* cfg, const wm_cache* cache, const wm_mix_weights* w,
                     const void* h, const int32_t* page_table, const int32_t* slot, int32_t B,

@@ -277,20 +277,28 @@ __global__ void __launch_bounds__(kThreads, attn_ctas_per_sm(SB, G)) decode_attn
       lens[i] = ok ? S : 0;
       sum += ok ? (S + STAGE_SLOTS - 1) / STAGE_SLOTS : 0;
     }
-    scan[tid] = sum;
-    __syncthreads();
-    for (int o = 1; o < kThreads; o <<= 1) {  // inclusive Hillis-Steele scan
-      const int v = tid >= o ? scan[tid - o] : 0;
-      __syncthreads();
-      scan[tid] += v;
-      __syncthreads();
+    // exclusive prefix sum over the block: shuffles within each warp, then
+    // the warp totals (one barrier instead of one per doubling step)
+    int incl = sum;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int v = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+      if (lane >= o) incl += v;
     }
-    int run = scan[tid] - sum;
+    if (lane == 31) scan[warp] = incl;
+    __syncthreads();
+    int before = 0, total = 0;
+#pragma unroll
+    for (int w = 0; w < kWarps; ++w) {
+      before += w < warp ? scan[w] : 0;
+      total += scan[w];
+    }
+    int run = before + incl - sum;
     for (int i = i0; i < i1; ++i) {
       pre[i] = run;
       run += lens[i] ? (lens[i] + STAGE_SLOTS - 1) / STAGE_SLOTS : 0;
     }
-    if (tid == kThreads - 1) pre[B] = scan[tid];
+    if (tid == kThreads - 1) pre[B] = total;
     if (lane == 0) {
       for (int s = 0; s < kWStages; ++s) mbar_init(&bars[warp][s], 1);
       mbar_init(&qbars[warp], 1);

@@ -81,6 +81,12 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   uint8_t* As = base;
   uint8_t* Bs = base + NS * a_bytes;
 
+  constexpr int HPT = kTcM / HD;  // whole heads per 128-row tile
+  const int wrow = MODE == kEpiKV ? j * p.M_item + mt * HPT * HD : mt * kTcM;
+  const int xrow = (MODE == kEpiKV ? (X * p.k + j) * p.B : X * p.B) + n0;
+  const int kb0 = MODE == kEpiKV ? 0 : j * p.kb_per_split;
+  const int kb1 = MODE == kEpiKV ? p.nk : min(p.nk, kb0 + p.kb_per_split);
+  const int nkb = kb1 - kb0;
   if (threadIdx.x == 0) {
     for (int s = 0; s < NS; ++s) {
       mbar_init(&full[s], 1);
@@ -90,8 +96,16 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     fence_mbar_init();
     tc::prefetch_tensormap(tmW);
     tc::prefetch_tensormap(&tmX);
+    // The weights are inputs no earlier kernel writes: the first ring's worth
+    // streams in while the previous grid finishes.  Each stage's barrier
+    // expects these bytes now and completes only after the arrival that
+    // comes with the activation tile, after the dependency wait.
+    for (int kb = 0; kb < NS && kb < nkb; ++kb) {
+      mbar_expect_tx(&full[kb], a_bytes);
+      tc::tma_load_2d(As + kb * a_bytes, tmW, (kb0 + kb) * kTcBK, wrow, &full[kb]);
+    }
   }
-  // programmatic dependent launch: inputs may come from the previous grid
+  // programmatic dependent launch: the activations come from the previous grid
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   asm volatile("griddepcontrol.wait;" ::: "memory");
   float* rope_s = reinterpret_cast<float*>(base + p.rope_smem_off);  // [B][HD/2][2] or unused
@@ -103,18 +117,18 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   __syncthreads();
   tc::fence_after_sync();
   const uint32_t tmem = tmem_base;
-  constexpr int HPT = kTcM / HD;  // whole heads per 128-row tile
-  const int wrow = MODE == kEpiKV ? j * p.M_item + mt * HPT * HD : mt * kTcM;
-  const int xrow = (MODE == kEpiKV ? (X * p.k + j) * p.B : X * p.B) + n0;
-  const int kb0 = MODE == kEpiKV ? 0 : j * p.kb_per_split;
-  const int kb1 = MODE == kEpiKV ? p.nk : min(p.nk, kb0 + p.kb_per_split);
-  const int nkb = kb1 - kb0;
 
   if (warp == 0 && lane == 0) {
-    // TMA producer
+    // TMA producer: activation tiles for the prefetched stages, then whole
+    // stages as the ring frees up
     for (int kb = 0; kb < nkb; ++kb) {
       const int s = kb % NS;
-      if (kb >= NS && !mbar_wait(&empty[s], ((kb / NS) - 1) & 1)) {
+      if (kb < NS) {
+        mbar_arrive_expect_tx(&full[s], b_bytes);
+        tc::tma_load_2d(Bs + s * b_bytes, &tmX, (kb0 + kb) * kTcBK, xrow, &full[s]);
+        continue;
+      }
+      if (!mbar_wait(&empty[s], ((kb / NS) - 1) & 1)) {
         report(p.status, WM_ERR_TIMEOUT);
         break;
       }

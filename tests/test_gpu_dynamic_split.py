@@ -4,10 +4,10 @@ every output row against the fp64 oracle.
 Launches reading 2 GB of K/V or more cut the KV stream into about eight
 chunks per warp and hand them out from a device counter; units crossing
 chunk boundaries leave partial records that the piece completing the unit
-merges.  Small launches take that path under WM_ATTN_DYNAMIC_SPLIT, so the
-first tests cover many chunk boundaries per unit on shapes the oracle checks
-in full; the last ones run whole full-size layers of the two largest
-workloads, where the path is taken by default, and compare every row.
+merges.  Small launches take that path under WM_ATTN_DYNAMIC_SPLIT, so these
+tests cover many chunk boundaries per unit on shapes the oracle checks in
+full; whole full-size layers, where the path is taken by default, are
+compared row by row in test_gpu_full_size.py.
 """
 import numpy as np
 import pytest
@@ -88,23 +88,3 @@ def test_dynamic_split_repeated_launches_leave_no_stale_state():
         assert H.rel_err(H.to_f64(out), want[:B]) <= H.TOL[w.dtype], B
     assert sess.read_status() == 0
     _free()
-
-
-@pytest.mark.parametrize("name,layer", [("large", 13), ("long128k", 5)])
-def test_full_size_layer_every_row(name, layer):
-    """One whole layer of the full-size workload (3.3 GB and 17.2 GB of K/V
-    per launch), every (sequence, query head) row against the oracle."""
-    w = configs.get(name)
-    prob, sess, dp = H.setup(w)
-    plan = W.wm_decode_attn_plan(sess.cfg, w.B, prob.max_pages)
-    assert plan["chunk_stages"] > 0, plan  # the dynamic path, taken by default
-    assert _stages(w, prob.seq_lens) // plan["chunk_stages"] > plan["warps"], plan
-    out = H.run_attn(sess, dp, layer)
-    torch.cuda.synchronize()
-    assert sess.read_status() == 0
-    got = H.to_f64(out)
-    del sess, dp, out
-    _free()
-    want = H.oracle_attn_layer(prob, layer)
-    err_rows = np.abs(got - want).max(axis=2) / np.abs(want).max()
-    assert float(err_rows.max()) <= H.TOL[w.dtype], np.unravel_index(err_rows.argmax(), err_rows.shape)

@@ -295,8 +295,12 @@ __global__ void __launch_bounds__(256) gemm_wxT_simt(const GemmArgs a) {
 // ---------------------------------------------------------------- mix
 // One CTA per (token, branch, group of kChanGroup channels).  Thread t owns
 // the 8-element vectors t, t + 256 of D, so h, gains and the output move as
-// 16-byte vectors.
-template <typename T>
+// 16-byte vectors.  PRE (decode shapes: L <= kMixPreL, D <= 8 * 256): the
+// thread's h vectors of every layer and its gains are loaded before the
+// router partials are summed, so the kernel waits for one round of loads.
+constexpr int kMixPreL = 16;
+
+template <typename T, bool PRE>
 __global__ void __launch_bounds__(kMixThreads) mix_kernel(const MixParams p) {
   extern __shared__ float sm[];  // alpha[kChanGroup][L], r[L]
   __shared__ float red[kMixThreads / 32][kChanGroup];
@@ -306,7 +310,24 @@ __global__ void __launch_bounds__(kMixThreads) mix_kernel(const MixParams p) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int nj = min(kChanGroup, p.k - j0);
   const int kL = p.k * p.L;
+  const int nvec = p.D / 8;
+  const T* hp = reinterpret_cast<const T*>(p.h) + (int64_t)b * p.L * p.D;
+  const T* g = reinterpret_cast<const T*>(p.pre_g[X]);
   pdl_wait();
+  // PRE: this thread's vector of every layer, of the pre-mix gain and of the
+  // channel gains, all in flight before the router partials are read
+  uint4 hpre[PRE ? kMixPreL : 1], gpre, cpre[kChanGroup];
+  if (PRE && tid < nvec) {
+#pragma unroll
+    for (int l = 0; l < (PRE ? kMixPreL : 1); ++l)
+      if (l < p.L) hpre[l] = __ldg(reinterpret_cast<const uint4*>(hp + (int64_t)l * p.D + tid * 8));
+    gpre = __ldg(reinterpret_cast<const uint4*>(g + tid * 8));
+#pragma unroll
+    for (int jj = 0; jj < kChanGroup; ++jj)
+      if (jj < nj)
+        cpre[jj] = __ldg(reinterpret_cast<const uint4*>(reinterpret_cast<const T*>(p.ch_g[X]) +
+                                                        (int64_t)(j0 + jj) * p.D + tid * 8));
+  }
   const T* br = reinterpret_cast<const T*>(p.br[X]);
   // alpha[j][l] = z[j*L + l] = bias + sum of the router's split partials
   for (int i = tid; i < nj * p.L; i += kMixThreads) {
@@ -320,37 +341,59 @@ __global__ void __launch_bounds__(kMixThreads) mix_kernel(const MixParams p) {
   for (int i = tid; i < p.L; i += kMixThreads) rl[i] = p.inv_rms[b * p.L + i];
   __syncthreads();
 
-  const int nvec = p.D / 8;
-  const T* hp = reinterpret_cast<const T*>(p.h) + (int64_t)b * p.L * p.D;
-  const T* g = reinterpret_cast<const T*>(p.pre_g[X]);
   float gv[kVecPerThread][8];
   float acc[kChanGroup][kVecPerThread][8];
 #pragma unroll
   for (int v = 0; v < kVecPerThread; ++v) {
     const int vi = tid + v * kMixThreads;
-    if (vi < nvec) load8f<T>(g + vi * 8, gv[v]);
+    if (PRE) {
+      if (v == 0 && vi < nvec) Elem<T>::unpack(gpre, gv[0]);
+    } else if (vi < nvec) {
+      load8f<T>(g + vi * 8, gv[v]);
+    }
 #pragma unroll
     for (int jj = 0; jj < kChanGroup; ++jj)
 #pragma unroll
       for (int i = 0; i < 8; ++i) acc[jj][v][i] = 0.f;
   }
-#pragma unroll 4
-  for (int l = 0; l < p.L; ++l) {
-    const float r = rl[l];
-    float a[kChanGroup];
+  if (PRE) {
+    if (tid < nvec) {
 #pragma unroll
-    for (int jj = 0; jj < kChanGroup; ++jj) a[jj] = jj < nj ? alpha[jj * p.L + l] : 0.f;
+      for (int l = 0; l < (PRE ? kMixPreL : 1); ++l) {
+        if (l >= p.L) break;
+        const float r = rl[l];
+        float a[kChanGroup];
 #pragma unroll
-    for (int v = 0; v < kVecPerThread; ++v) {
-      const int vi = tid + v * kMixThreads;
-      if (vi < nvec) {
+        for (int jj = 0; jj < kChanGroup; ++jj) a[jj] = jj < nj ? alpha[jj * p.L + l] : 0.f;
         float hv[8];
-        load8f<T>(hp + (int64_t)l * p.D + vi * 8, hv);
+        Elem<T>::unpack(hpre[l], hv);
 #pragma unroll
         for (int i = 0; i < 8; ++i) {
-          const float hh = hv[i] * r * gv[v][i];  // pre-mix RMSNorm with gain
+          const float hh = hv[i] * r * gv[0][i];  // pre-mix RMSNorm with gain
 #pragma unroll
-          for (int jj = 0; jj < kChanGroup; ++jj) acc[jj][v][i] = fmaf(a[jj], hh, acc[jj][v][i]);
+          for (int jj = 0; jj < kChanGroup; ++jj) acc[jj][0][i] = fmaf(a[jj], hh, acc[jj][0][i]);
+        }
+      }
+    }
+  } else {
+#pragma unroll 4
+    for (int l = 0; l < p.L; ++l) {
+      const float r = rl[l];
+      float a[kChanGroup];
+#pragma unroll
+      for (int jj = 0; jj < kChanGroup; ++jj) a[jj] = jj < nj ? alpha[jj * p.L + l] : 0.f;
+#pragma unroll
+      for (int v = 0; v < kVecPerThread; ++v) {
+        const int vi = tid + v * kMixThreads;
+        if (vi < nvec) {
+          float hv[8];
+          load8f<T>(hp + (int64_t)l * p.D + vi * 8, hv);
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            const float hh = hv[i] * r * gv[v][i];  // pre-mix RMSNorm with gain
+#pragma unroll
+            for (int jj = 0; jj < kChanGroup; ++jj) acc[jj][v][i] = fmaf(a[jj], hh, acc[jj][v][i]);
+          }
         }
       }
     }
@@ -387,7 +430,10 @@ __global__ void __launch_bounds__(kMixThreads) mix_kernel(const MixParams p) {
       const int vi = tid + v * kMixThreads;
       if (vi < nvec) {
         float cv[8], o[8];
-        load8f<T>(cg + vi * 8, cv);
+        if (PRE)
+          Elem<T>::unpack(cpre[jj], cv);
+        else
+          load8f<T>(cg + vi * 8, cv);
 #pragma unroll
         for (int i = 0; i < 8; ++i) o[i] = acc[jj][v][i] * ss[jj] * cv[i];
         store8f<T>(xo + vi * 8, o);
@@ -666,7 +712,14 @@ cudaError_t launch_all(MixParams& p, cudaStream_t s) {
   } else {
     const size_t smem = sizeof(float) * (kChanGroup * p.L + p.L);
     dim3 grid(p.B, 2, (p.k + kChanGroup - 1) / kChanGroup);
-    e = launch_pdl(mix_kernel<T>, grid, dim3(kMixThreads), smem, s, p);
+    bool pre = false;  // bf16 decode shapes: every load issued up front
+    if constexpr (sizeof(T) == 2) pre = p.L <= kMixPreL && p.D / 8 <= kMixThreads;
+    if constexpr (sizeof(T) == 2) {
+      e = pre ? launch_pdl(mix_kernel<T, true>, grid, dim3(kMixThreads), smem, s, p)
+              : launch_pdl(mix_kernel<T, false>, grid, dim3(kMixThreads), smem, s, p);
+    } else {
+      e = launch_pdl(mix_kernel<T, false>, grid, dim3(kMixThreads), smem, s, p);
+    }
     if (e != cudaSuccess) return e;
   }
   if (bf16 && proj_tc_supported(p)) {

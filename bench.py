@@ -54,10 +54,18 @@ def measured_peak():
 
 def kernel_source_hash() -> str:
     h = hashlib.sha256()
-    for f in ("attn.cu", "attn_kernel.cuh", "attn_bf16.cu", "common.cuh", "internal.h", "wm_api.cu"):
+    for f in ("attn.cu", "attn_kernel.cuh", "attn_bf16.cu", "attn_unit.cuh", "attn_unit_bf16.cu",
+              "common.cuh", "internal.h", "wm_api.cu"):
         with open(os.path.join(ROOT, "paper_2608_18486_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:16]
+
+
+def attn_kernel_name(cfg, w, prob) -> str:
+    """The decode-attention kernel the library's planner picks for this launch."""
+    from paper_2608_18486_gb300 import _lib as W
+    plan = W.wm_decode_attn_plan(cfg, w.B, prob.max_pages)
+    return "decode_attn_unit_kernel" if plan["unit_ctas"] > 0 else "decode_attn_kernel"
 
 
 def ncu_traffic(workload: str):
@@ -477,7 +485,7 @@ def run_gpu(args, w):
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms / args.steps,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": w.dtype,
             "data": "synthetic", "config": config_dict(w, world),
-            "roofline": {"bound": "hbm", "kernel": "decode_attn_kernel", "achieved": achieved,
+            "roofline": {"bound": "hbm", "kernel": attn_kernel_name(cfg, w, prob), "achieved": achieved,
                          "peak": peak, "peak_kind": peak_kind, "unit": "GB/s",
                          "frac": achieved / peak, "traffic": traffic,
                          "algorithmic_bytes_per_launch": launch_bytes,

@@ -204,6 +204,7 @@ wm_status wm_decode_attn(const wm_config* cfg, const wm_cache* cache, int32_t la
 /* Flags of wm_decode_attn_flags. */
 #define WM_ATTN_INPUTS_READY 1u
 #define WM_ATTN_DYNAMIC_SPLIT 2u
+#define WM_ATTN_UNIT_SPLIT 4u
 
 /*
  * wm_decode_attn with flags; wm_decode_attn(...) is wm_decode_attn_flags(...,
@@ -226,7 +227,17 @@ wm_status wm_decode_attn(const wm_config* cfg, const wm_cache* cache, int32_t la
  *     result is the same within rounding (the merge order of the pieces of
  *     a unit depends on where the chunks end, not on which warp takes them).
  *     wm_decode_attn_workspace covers either split.
- * Unknown flag bits return WM_ERR_INVALID_ARG.
+ *   WM_ATTN_UNIT_SPLIT: give every (sequence, kv head) unit one cluster of
+ *     C = min(8, max(1, SMs / units)) CTAs whose warps each stream an equal
+ *     share of the unit and merge on chip (shared and distributed shared
+ *     memory), whatever the launch size.  Without it the split is taken only
+ *     for launches below 2 GB where, at the largest C >= 2 whose clusters
+ *     are all resident at once, it runs at least 60% of the warps of the
+ *     static split above (the paper's model shape, 48 units: C = 2); every
+ *     other launch streams as above.  The unit split uses no workspace and
+ *     gives the same result within rounding.
+ * Unknown flag bits, or DYNAMIC_SPLIT together with UNIT_SPLIT, return
+ * WM_ERR_INVALID_ARG.
  */
 wm_status wm_decode_attn_flags(const wm_config* cfg, const wm_cache* cache, int32_t layer,
                                const void* q, const int32_t* page_table,
@@ -236,14 +247,15 @@ wm_status wm_decode_attn_flags(const wm_config* cfg, const wm_cache* cache, int3
 
 /*
  * How wm_decode_attn_flags would split a launch (no GPU work; for tuning and
- * tests).  Fills plan[0..3] with: the persistent grid (CTAs), warps in it,
- * work chunks it cuts the KV stream into at most, and stages (8 KB of K+V)
- * per chunk, 0 meaning a static split with one chunk per warp.  The chunk
- * count of a static split is its warp count.  Returns WM_ERR_INVALID_ARG for
- * a bad config, B < 1, max_pages < 1, unknown flags or plan == NULL.
+ * tests).  Fills plan[0..4] with: the grid (CTAs), warps in it, work
+ * chunks a stream-K launch cuts the KV stream into at most, stages (8 KB of
+ * K+V) per chunk (0: a static split, one chunk per warp, whose chunk count is
+ * its warp count), and the CTAs per unit of the unit split (0: stream-K; then
+ * the grid is persistent).  Returns WM_ERR_INVALID_ARG for a bad config,
+ * B < 1, max_pages < 1, unknown or conflicting flags, or plan == NULL.
  */
 wm_status wm_decode_attn_plan(const wm_config* cfg, int32_t B, int32_t max_pages, uint32_t flags,
-                              int32_t plan[4]);
+                              int32_t plan[5]);
 
 /*
  * Causal channel attention of one layer for many query positions at once:

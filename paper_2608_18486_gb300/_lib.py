@@ -22,6 +22,7 @@ EXPORTED = ["wm_status_string", "wm_config_check", "wm_cache_bytes", "wm_cache_a
             "wm_kv_mix_launches"]
 WM_ATTN_INPUTS_READY = 1
 WM_ATTN_DYNAMIC_SPLIT = 2
+WM_ATTN_UNIT_SPLIT = 4
 
 
 class wm_config(ctypes.Structure):
@@ -184,12 +185,14 @@ def wm_kv_mix_launches(cfg, B) -> int:
 
 
 def wm_decode_attn_plan(cfg, B, max_pages, flags=0) -> dict:
-    """How a launch would be split: grid, warps, chunks, stages per chunk."""
-    plan = (ctypes.c_int32 * 4)()
+    """How a launch would be split: grid, warps, chunks, stages per chunk,
+    CTAs per unit of the unit split (0: stream-K)."""
+    plan = (ctypes.c_int32 * 5)()
     rc = lib().wm_decode_attn_plan(ctypes.byref(cfg), int(B), int(max_pages), int(flags), plan)
     if rc != WM_OK:
         raise WMError(rc, "wm_decode_attn_plan")
-    return {"grid": plan[0], "warps": plan[1], "chunks": plan[2], "chunk_stages": plan[3]}
+    return {"grid": plan[0], "warps": plan[1], "chunks": plan[2], "chunk_stages": plan[3],
+            "unit_ctas": plan[4]}
 
 
 def wm_prefill_attn(cfg, cache, layer, q, pos, page_table, B, Tq, max_pages, out, dev_status,

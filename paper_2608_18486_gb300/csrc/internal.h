@@ -50,6 +50,14 @@ int attn_warps_per_cta();
 size_t attn_smem_bytes(int stage_bytes, int dtype, int d, int G, int B);
 cudaError_t launch_decode_attn(const AttnParams& p, int stage_bytes, int dtype, int d, int G,
                                int grid, cudaStream_t s);
+// Unit split (attn_unit.cuh): one cluster of `cluster` CTAs (<= 8) per
+// (sequence, kv head) unit, `units` = B * Hkv clusters.
+constexpr int kAttnUnitMaxCluster = 8;
+int attn_unit_warps_per_cta(int stage_bytes, int dtype, int d, int G);  // 0: unsupported
+size_t attn_unit_smem_bytes(int stage_bytes, int dtype, int d, int G);
+int attn_unit_max_clusters(int stage_bytes, int dtype, int d, int G, int cluster);
+cudaError_t launch_decode_attn_unit(const AttnParams& p, int stage_bytes, int dtype, int d, int G,
+                                    int units, int cluster, cudaStream_t s);
 
 // ------------------------------------------------------------ prefill attention
 struct PrefillLaunch {

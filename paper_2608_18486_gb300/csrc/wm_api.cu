@@ -39,10 +39,12 @@ bool aligned(const void* p, size_t a) { return ((uintptr_t)p % a) == 0; }
 // Persistent grid of one attention launch and its workspace layout.
 struct AttnPlan {
   int stage_bytes, grid, nwarps, chunk_stages, max_chunks;
+  int unit_ctas;  // > 0: unit split, one cluster of this many CTAs per unit
   size_t off_part, off_counters, total;
 };
 
 constexpr int kAttnMaxBatch = 4096;
+constexpr uint32_t kAttnFlags = WM_ATTN_INPUTS_READY | WM_ATTN_DYNAMIC_SPLIT | WM_ATTN_UNIT_SPLIT;
 // K + V bytes of one pipeline stage: 8 KB, 2 CTAs (8 warps) per SM.  A warp
 // spends about as long on the bookkeeping of a stage (wait, copy issue,
 // piece checks) as on its math, so 4 KB stages at 4 CTAs per SM were
@@ -72,12 +74,43 @@ constexpr int kAttnMinStagesPerWarp = 4;
 // A static split has at most one chunk per warp; a dynamic one chunks of
 // ceil(NS / (warps * kAttnChunksPerWarp)) stages or more, so at most
 // warps * kAttnChunksPerWarp of them.
+// Unit split (one cluster of C CTAs per (sequence, kv head) unit, merged on
+// chip) instead of a static stream-K split when, with the largest C >= 2 at
+// which every cluster is resident at once, it runs at least this share of
+// the stream-K grid's warps.  Its merge costs a fraction of stream-K's
+// cross-SM one, so it wins even on fewer SMs: on the paper's model shape (48
+// units; clusters of 3 do not all fit) 96 SMs of 12 warps took 10.9 us per
+// launch against 17.4 us for stream-K on all 152.  It is static, so it
+// suits units of similar length, which the small launches of one decode
+// step have.
+constexpr double kAttnUnitMinWarpShare = 0.6;
+
+// Resident clusters of C unit-split CTAs for (dtype, d, G) on this device,
+// cached (0: unknown or no device).
+int unit_max_clusters(int dtype, int d, int G, int C) {
+  static std::atomic<int> cache[kMaxDevices][2][3][4][wm::kAttnUnitMaxCluster + 1];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return 0;
+  const int di = d == 64 ? 0 : d == 96 ? 1 : d == 128 ? 2 : -1;
+  const int gi = G == 1 ? 0 : G == 2 ? 1 : G == 4 ? 2 : G == 8 ? 3 : -1;
+  if (di < 0 || gi < 0 || C < 1 || C > wm::kAttnUnitMaxCluster) return 0;
+  std::atomic<int>& slot = cache[dev][dtype == WM_DT_F32 ? 1 : 0][di][gi][C];
+  int v = slot.load(std::memory_order_relaxed);
+  if (v == 0) {
+    v = 1 + wm::attn_unit_max_clusters(kAttnStageBytes, dtype, d, G, C);
+    slot.store(v, std::memory_order_relaxed);
+  }
+  return v - 1;
+}
+
 int64_t attn_chunk_capacity() {
   return (int64_t)sm_count() * wm::attn_ctas_per_sm(kAttnStageBytes, 1) * wm::attn_warps_per_cta() *
          kAttnChunksPerWarp;
 }
 
-AttnPlan attn_plan(const wm_config& c, int32_t B, int32_t max_pages, bool force_dynamic = false) {
+AttnPlan attn_plan(const wm_config& c, int32_t B, int32_t max_pages, uint32_t flags = 0) {
+  const bool force_dynamic = (flags & WM_ATTN_DYNAMIC_SPLIT) != 0;
+  const bool force_unit = (flags & WM_ATTN_UNIT_SPLIT) != 0;
   AttnPlan pl{};
   const int64_t max_slots = (int64_t)max_pages * c.page_size;
   const double kv_bytes = (double)B * c.Hkv * max_slots * 2.0 * c.d * elem_size(c.dtype);
@@ -118,6 +151,26 @@ AttnPlan attn_plan(const wm_config& c, int32_t B, int32_t max_pages, bool force_
   pl.off_part = off;
   off += align256(sizeof(float) * 2 * (size_t)pl.max_chunks * wm::attn_part_rec(G, c.d));
   pl.total = off;
+  // the unit split (it needs no workspace; the stream-K layout above stays
+  // the size the workspace query reports)
+  const int64_t units = (int64_t)B * c.Hkv;
+  const int nsm = sm_count();
+  const int unit_warps = wm::attn_unit_warps_per_cta(pl.stage_bytes, c.dtype, c.d, G);
+  if (force_unit) {
+    int64_t C = nsm / units;
+    pl.unit_ctas = (int)(C < 1 ? 1 : C > wm::kAttnUnitMaxCluster ? wm::kAttnUnitMaxCluster : C);
+  } else if (!force_dynamic && pl.chunk_stages == 0 && unit_warps > 0) {
+    for (int C = wm::kAttnUnitMaxCluster; C >= 2; --C) {
+      if (units * C > nsm || unit_max_clusters(c.dtype, c.d, G, C) < units) continue;
+      if ((double)(units * C * unit_warps) >= kAttnUnitMinWarpShare * pl.nwarps) pl.unit_ctas = C;
+      break;
+    }
+  }
+  if (pl.unit_ctas > 0) {
+    pl.grid = (int)(units * pl.unit_ctas);
+    pl.nwarps = pl.grid * unit_warps;
+    pl.chunk_stages = 0;
+  }
   return pl;
 }
 
@@ -168,7 +221,8 @@ wm_status decode_attn_impl(const wm_config* c, const wm_cache* cache, int32_t la
                            void* stream) {
   wm_status st = wm_config_check(c);
   if (st != WM_OK) return st;
-  if (flags & ~(uint32_t)(WM_ATTN_INPUTS_READY | WM_ATTN_DYNAMIC_SPLIT)) return WM_ERR_INVALID_ARG;
+  if (flags & ~kAttnFlags) return WM_ERR_INVALID_ARG;
+  if ((flags & WM_ATTN_DYNAMIC_SPLIT) && (flags & WM_ATTN_UNIT_SPLIT)) return WM_ERR_INVALID_ARG;
   if ((st = check_cache(*c, cache)) != WM_OK) return st;
   if (layer < 0 || layer >= c->L || B < 0 || max_pages < 1) return WM_ERR_INVALID_ARG;
   if ((int64_t)max_pages * c->page_size > INT32_MAX / 2) return WM_ERR_INVALID_ARG;
@@ -177,7 +231,7 @@ wm_status decode_attn_impl(const wm_config* c, const wm_cache* cache, int32_t la
   if ((int64_t)B * c->Hq > INT32_MAX / 2) return WM_ERR_UNSUPPORTED;  // 32-bit output rows
   if (!q || !page_table || !seq_lens || !out || !workspace) return WM_ERR_INVALID_ARG;
   if (!aligned(q, 16) || !aligned(out, 16) || !aligned(workspace, 256)) return WM_ERR_INVALID_ARG;
-  const AttnPlan pl = attn_plan(*c, B, max_pages, (flags & WM_ATTN_DYNAMIC_SPLIT) != 0);
+  const AttnPlan pl = attn_plan(*c, B, max_pages, flags);
   if (ws_bytes < pl.total) return WM_ERR_INVALID_ARG;
   if (pl.max_chunks > attn_chunk_capacity()) return WM_ERR_UNSUPPORTED;  // cannot happen
 
@@ -210,8 +264,12 @@ wm_status decode_attn_impl(const wm_config* c, const wm_cache* cache, int32_t la
   if (clear_workspace &&
       cudaMemsetAsync(workspace, 0, pl.total, (cudaStream_t)stream) != cudaSuccess)
     return WM_ERR_CUDA;
-  cudaError_t e = wm::launch_decode_attn(p, pl.stage_bytes, c->dtype, c->d, c->Hq / c->Hkv,
-                                         pl.grid, (cudaStream_t)stream);
+  cudaError_t e =
+      pl.unit_ctas > 0
+          ? wm::launch_decode_attn_unit(p, pl.stage_bytes, c->dtype, c->d, c->Hq / c->Hkv,
+                                        B * c->Hkv, pl.unit_ctas, (cudaStream_t)stream)
+          : wm::launch_decode_attn(p, pl.stage_bytes, c->dtype, c->d, c->Hq / c->Hkv, pl.grid,
+                                   (cudaStream_t)stream);
   return e == cudaSuccess ? WM_OK : WM_ERR_CUDA;
 }
 
@@ -278,20 +336,22 @@ size_t wm_decode_attn_workspace(const wm_config* c, int32_t B, int32_t max_pages
   if (wm_config_check(c) != WM_OK || B < 0 || max_pages < 1) return 0;
   if (B == 0) return 256;
   // enough for either split (WM_ATTN_DYNAMIC_SPLIT may cut more chunks)
-  const size_t a = attn_plan(*c, B, max_pages, false).total;
-  const size_t b = attn_plan(*c, B, max_pages, true).total;
+  const size_t a = attn_plan(*c, B, max_pages, 0u).total;
+  const size_t b = attn_plan(*c, B, max_pages, WM_ATTN_DYNAMIC_SPLIT).total;
   return a > b ? a : b;
 }
 
 wm_status wm_decode_attn_plan(const wm_config* c, int32_t B, int32_t max_pages, uint32_t flags,
-                              int32_t plan[4]) {
+                              int32_t plan[5]) {
   if (wm_config_check(c) != WM_OK || B < 1 || max_pages < 1 || !plan) return WM_ERR_INVALID_ARG;
-  if (flags & ~(uint32_t)(WM_ATTN_INPUTS_READY | WM_ATTN_DYNAMIC_SPLIT)) return WM_ERR_INVALID_ARG;
-  const AttnPlan pl = attn_plan(*c, B, max_pages, (flags & WM_ATTN_DYNAMIC_SPLIT) != 0);
+  if (flags & ~kAttnFlags) return WM_ERR_INVALID_ARG;
+  if ((flags & WM_ATTN_DYNAMIC_SPLIT) && (flags & WM_ATTN_UNIT_SPLIT)) return WM_ERR_INVALID_ARG;
+  const AttnPlan pl = attn_plan(*c, B, max_pages, flags);
   plan[0] = pl.grid;
   plan[1] = pl.nwarps;
   plan[2] = pl.max_chunks;
   plan[3] = pl.chunk_stages;
+  plan[4] = pl.unit_ctas;
   return WM_OK;
 }
 

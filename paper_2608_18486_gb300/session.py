@@ -62,14 +62,18 @@ class DecodeSession:
 
     # ------------------------------------------------------------------ calls
     def decode_attn(self, layer: int, q, page_table, seq_lens, out, B: int | None = None,
-                    stream=None, inputs_ready: bool = False, dynamic_split: bool = False) -> None:
+                    stream=None, inputs_ready: bool = False, dynamic_split: bool = False,
+                    unit_split: bool = False) -> None:
         """inputs_ready: the previous work on the stream wrote no cache, page
         table, lengths or workspace (true for layers 1..L-1 of a decode step).
         dynamic_split: chunks handed out by a device counter whatever the
-        launch size (WM_ATTN_DYNAMIC_SPLIT)."""
+        launch size (WM_ATTN_DYNAMIC_SPLIT).  unit_split: one cluster of CTAs
+        per (sequence, kv head) unit whatever the launch size
+        (WM_ATTN_UNIT_SPLIT)."""
         B = self.B if B is None else B
         flags = (W.WM_ATTN_INPUTS_READY if inputs_ready else 0) | \
-            (W.WM_ATTN_DYNAMIC_SPLIT if dynamic_split else 0)
+            (W.WM_ATTN_DYNAMIC_SPLIT if dynamic_split else 0) | \
+            (W.WM_ATTN_UNIT_SPLIT if unit_split else 0)
         rc = W.wm_decode_attn_flags(self.cfg, self.cache, layer, q, page_table, seq_lens, B,
                                     self.max_pages, out, self.attn_ws, self.attn_ws_bytes, flags,
                                     self.status, self._stream(stream))

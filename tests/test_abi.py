@@ -102,8 +102,11 @@ def test_compute_calls_reject_bad_arguments_before_launching():
     # a cache laid out for another config is refused
     other = cfg(k=8)
     assert W.wm_decode_attn(other, cache, 0, fake, fake, fake, 2, 4, fake, fake, ws, None, None) == W.WM_ERR_INVALID_ARG
-    assert W.wm_decode_attn_flags(c, cache, 0, fake, fake, fake, 2, 4, fake, fake, ws, 4, None,
+    assert W.wm_decode_attn_flags(c, cache, 0, fake, fake, fake, 2, 4, fake, fake, ws, 8, None,
                                   None) == W.WM_ERR_INVALID_ARG  # unknown flag bit
+    both = W.WM_ATTN_DYNAMIC_SPLIT | W.WM_ATTN_UNIT_SPLIT  # two splits at once
+    assert W.wm_decode_attn_flags(c, cache, 0, fake, fake, fake, 2, 4, fake, fake, ws, both, None,
+                                  None) == W.WM_ERR_INVALID_ARG
     wts = W.mix_weights((fake, fake), (fake, fake), (fake, fake), (fake, fake), (fake, fake), fake)
     mws = W.wm_kv_mix_workspace(c, 2)
     assert W.wm_kv_mix(c, cache, wts, fake, fake, fake, 2, 4, fake, mws - 1, None, None) == W.WM_ERR_INVALID_ARG
@@ -186,7 +189,23 @@ def test_attention_plan_static_and_dynamic_split():
                        lw.chan_of_layer())
     big = W.wm_decode_attn_plan(lc, lw.B, -(-(lw.ctx + 1) // lw.page))
     assert big["chunk_stages"] > 0 and big["chunks"] > big["warps"]
+    assert st["unit_ctas"] == 0 and dy["unit_ctas"] == 0 and big["unit_ctas"] == 0
+    # the unit split: one cluster of C CTAs per (sequence, kv head) unit, C at
+    # most 8 and no more SMs than the device has (units > SMs: C = 1)
+    un = W.wm_decode_attn_plan(c, w.B, max_pages, W.WM_ATTN_UNIT_SPLIT)
+    assert un["unit_ctas"] == 1 and un["grid"] == w.B * w.Hkv and un["chunk_stages"] == 0
+    pw = configs.get("paper_k16")
+    pc = W.make_config(pw.L, pw.k, pw.D, pw.Hq, pw.Hkv, pw.d, pw.p, pw.page, pw.dtype,
+                       pw.chan_of_layer())
+    pmax = -(-(pw.ctx + 1) // pw.page)
+    pu = W.wm_decode_attn_plan(pc, pw.B, pmax, W.WM_ATTN_UNIT_SPLIT)
+    units = pw.B * pw.Hkv
+    assert 2 <= pu["unit_ctas"] <= 8 and pu["grid"] == units * pu["unit_ctas"]
+    assert pu["warps"] == 12 * pu["grid"]  # d = 96, G = 2: 12 warps per CTA
+    assert W.wm_decode_attn_plan(pc, 1, pmax, W.WM_ATTN_UNIT_SPLIT)["unit_ctas"] == 8
     with pytest.raises(W.WMError):
         W.wm_decode_attn_plan(c, w.B, max_pages, 8)  # unknown flag bit
+    with pytest.raises(W.WMError):
+        W.wm_decode_attn_plan(c, w.B, max_pages, W.WM_ATTN_DYNAMIC_SPLIT | W.WM_ATTN_UNIT_SPLIT)
     with pytest.raises(W.WMError):
         W.wm_decode_attn_plan(c, 0, max_pages)

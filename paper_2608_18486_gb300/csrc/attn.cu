@@ -46,7 +46,7 @@ size_t attn_unit_smem_bytes(int stage_bytes, int dtype, int d, int G) {
   const size_t esz = dtype == WM_DT_F32 ? 4 : 2;
   const size_t stage = (size_t)attn_stage_slots(stage_bytes, dtype, d) * 2 * d * esz;
   return (size_t)attn_unit_warps_per_cta(stage_bytes, dtype, d, G) * attn_unit_detail::kUStages * stage +
-         (size_t)(attn_unit_detail::unit_rec(G, d) + 3) / 4 * 4 * sizeof(float) + (size_t)G * d * esz;
+         (size_t)(attn_unit_detail::unit_rec(G, d) + 3) / 4 * 4 * sizeof(float);
 }
 
 int attn_unit_max_clusters(int stage_bytes, int dtype, int d, int G, int cluster) {

@@ -29,12 +29,32 @@ using attn_detail::SoftState;
 
 constexpr int kUStages = 3;  // ring depth per warp
 
-// Warps per CTA (one CTA per SM): 12 where their rings fit in shared memory
-// and their registers in the SM's 64K (stages of at most 6 KB, up to two
-// query heads per kv head: d = 96 bf16, the paper's head size), else 8.
+// Warps per CTA: 4 (three CTAs per SM) where stages are at most 6 KB and a
+// kv head has at most two query heads (d = 96, the paper's head size): the
+// smaller CTAs let clusters of 8 stay resident for its 48 units; else 8 (one
+// CTA per SM).
 template <typename T, int HD, int G, int SB>
 constexpr int unit_warps() {
-  return Shape<T, HD, SB>::STAGE_ELEMS * (int)sizeof(T) * 2 <= 6144 && G <= 2 ? 12 : 8;
+  return Shape<T, HD, SB>::STAGE_ELEMS * (int)sizeof(T) * 2 <= 6144 && G <= 2 ? 4 : 8;
+}
+// CTAs per SM the register budget is sized for (at most 12 warps of 170
+// registers per SM)
+constexpr int unit_min_blocks(int nw) { return nw <= 4 ? 3 : nw <= 6 ? 2 : 1; }
+
+// A row of global memory another grid may just have written, as the stage
+// math reads it (lane part lp owns 16-byte vectors lp, lp + LPS, ...), through
+// L2 (ld.global.cg): no stale L1 line can be read.
+template <typename T, int HD, int SB>
+__device__ __forceinline__ void load_row_l2(const T* row, int lp,
+                                            float2 (&f)[Shape<T, HD, SB>::EPL / 2]) {
+  using SH = Shape<T, HD, SB>;
+#pragma unroll
+  for (int v = 0; v < SH::NVL; ++v) {
+    float t[SH::VEC];
+    Elem<T>::unpack(__ldcg(reinterpret_cast<const uint4*>(row + (v * SH::LPS + lp) * SH::VEC)), t);
+#pragma unroll
+    for (int i = 0; i < SH::VEC / 2; ++i) f[v * SH::VEC / 2 + i] = make_float2(t[2 * i], t[2 * i + 1]);
+  }
 }
 
 // floats of one partial state: G x HD unnormalised outputs, then (max, sum)
@@ -42,14 +62,14 @@ constexpr int unit_warps() {
 constexpr int unit_rec(int G, int HD) { return G * HD + 2 * G; }
 
 template <typename T, int HD, int G, int SB>
-__global__ void __launch_bounds__(unit_warps<T, HD, G, SB>() * 32, 1)
+__global__ void __launch_bounds__(unit_warps<T, HD, G, SB>() * 32,
+                                  unit_min_blocks(unit_warps<T, HD, G, SB>()))
     decode_attn_unit_kernel(const AttnParams p) {
   using SH = Shape<T, HD, SB>;
   constexpr int NW = unit_warps<T, HD, G, SB>();
   constexpr int VEC = SH::VEC, LPS = SH::LPS, E2 = SH::EPL / 2;
   constexpr int STAGE_SLOTS = SH::STAGE_SLOTS, STAGE_ELEMS = SH::STAGE_ELEMS;
   constexpr uint32_t KV_BYTES = STAGE_ELEMS * sizeof(T);
-  constexpr uint32_t Q_BYTES = G * HD * sizeof(T);
   constexpr int E = G * HD;  // output elements of a unit
   constexpr int REC = unit_rec(G, HD);
   constexpr unsigned FULLMASK = 0xFFFFFFFFu;
@@ -59,9 +79,7 @@ __global__ void __launch_bounds__(unit_warps<T, HD, G, SB>() * 32, 1)
   extern __shared__ __align__(128) unsigned char smem_raw[];
   T* ring = reinterpret_cast<T*>(smem_raw);  // [NW][S][2][STAGE_ELEMS]
   float* crec = reinterpret_cast<float*>(ring + NW * kUStages * 2 * STAGE_ELEMS);  // [REC]
-  T* qs = reinterpret_cast<T*>(crec + (REC + 3) / 4 * 4);                       // [G][HD]
   __shared__ uint64_t bars[NW][kUStages];
-  __shared__ uint64_t qbar;
   __shared__ uint64_t masks[NW][kUStages];
 
   cg::cluster_group cluster = cg::this_cluster();
@@ -82,7 +100,6 @@ __global__ void __launch_bounds__(unit_warps<T, HD, G, SB>() * 32, 1)
   if (tid == 0) {
     for (int w = 0; w < NW; ++w)
       for (int s = 0; s < kUStages; ++s) mbar_init(&bars[w][s], 1);
-    mbar_init(&qbar, 1);
   }
   fence_mbar_init();
   __syncthreads();
@@ -167,11 +184,6 @@ __global__ void __launch_bounds__(unit_warps<T, HD, G, SB>() * 32, 1)
   int issued = 0;
   for (; issued < nmine && issued < kUStages; ++issued) issue(s0 + issued);
   if (early) asm volatile("griddepcontrol.wait;" ::: "memory");
-  if (tid == 0) {  // the unit's G query rows, shared by the CTA's warps
-    mbar_arrive_expect_tx(&qbar, Q_BYTES);
-    bulk_g2s(qs, reinterpret_cast<const T*>(p.q) + ((int64_t)b * p.Hq + h * G) * HD, Q_BYTES, &qbar,
-             policy);
-  }
 
   // ---- stream this warp's stages
   const int lane_slot = lane / LPS, lane_part = lane % LPS;
@@ -186,15 +198,14 @@ __global__ void __launch_bounds__(unit_warps<T, HD, G, SB>() * 32, 1)
 #pragma unroll
     for (int i = 0; i < E2; ++i) st.acc[g][i] = make_float2(0.f, 0.f);
   }
-  // warp 0 always waits for the query copy, so that no copy into this CTA's
-  // shared memory is in flight when it exits
-  bool alive = true;
-  if (nmine > 0 || warp == 0) alive = __all_sync(FULLMASK, mbar_wait(&qbar, 0));
-  if (!alive && lane == 0) report(p.status, WM_ERR_TIMEOUT);
-  if (nmine > 0 && alive) {
+  // the unit's G query rows, read through L2 after the dependency wait (the
+  // previous grid may have written them)
+  if (nmine > 0) {
+    const T* qrow = reinterpret_cast<const T*>(p.q) + ((int64_t)b * p.Hq + h * G) * HD;
 #pragma unroll
-    for (int g = 0; g < G; ++g) attn_detail::load_row<T, HD, SB>(qs + g * HD, lane_part, q2[g]);
+    for (int g = 0; g < G; ++g) load_row_l2<T, HD, SB>(qrow + g * HD, lane_part, q2[g]);
   }
+  bool alive = true;
   int done = 0;  // stages consumed
   for (; done < nmine && alive; ++done) {
     const int buf = done % kUStages;

@@ -161,7 +161,7 @@ AttnPlan attn_plan(const wm_config& c, int32_t B, int32_t max_pages, uint32_t fl
     pl.unit_ctas = (int)(C < 1 ? 1 : C > wm::kAttnUnitMaxCluster ? wm::kAttnUnitMaxCluster : C);
   } else if (!force_dynamic && pl.chunk_stages == 0 && unit_warps > 0) {
     for (int C = wm::kAttnUnitMaxCluster; C >= 2; --C) {
-      if (units * C > nsm || unit_max_clusters(c.dtype, c.d, G, C) < units) continue;
+      if (unit_max_clusters(c.dtype, c.d, G, C) < units) continue;
       if ((double)(units * C * unit_warps) >= kAttnUnitMinWarpShare * pl.nwarps) pl.unit_ctas = C;
       break;
     }

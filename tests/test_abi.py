@@ -201,7 +201,7 @@ def test_attention_plan_static_and_dynamic_split():
     pu = W.wm_decode_attn_plan(pc, pw.B, pmax, W.WM_ATTN_UNIT_SPLIT)
     units = pw.B * pw.Hkv
     assert 2 <= pu["unit_ctas"] <= 8 and pu["grid"] == units * pu["unit_ctas"]
-    assert pu["warps"] == 12 * pu["grid"]  # d = 96, G = 2: 12 warps per CTA
+    assert pu["warps"] == 4 * pu["grid"]  # d = 96, G = 2: 4 warps per CTA
     assert W.wm_decode_attn_plan(pc, 1, pmax, W.WM_ATTN_UNIT_SPLIT)["unit_ctas"] == 8
     with pytest.raises(W.WMError):
         W.wm_decode_attn_plan(c, w.B, max_pages, 8)  # unknown flag bit

@@ -29,13 +29,13 @@ using attn_detail::SoftState;
 
 constexpr int kUStages = 3;  // ring depth per warp
 
-// Warps per CTA: 4 (three CTAs per SM) where stages are at most 6 KB and a
-// kv head has at most two query heads (d = 96, the paper's head size): the
-// smaller CTAs let clusters of 8 stay resident for its 48 units; else 8 (one
-// CTA per SM).
+// Warps per CTA: 4 where a kv head has at most two query heads (two or
+// three CTAs per SM, by the stage size: smaller CTAs keep more clusters
+// resident and more SMs busy), else 8 (one CTA per SM: the states of four or
+// eight query heads take up to 255 registers).
 template <typename T, int HD, int G, int SB>
 constexpr int unit_warps() {
-  return Shape<T, HD, SB>::STAGE_ELEMS * (int)sizeof(T) * 2 <= 6144 && G <= 2 ? 4 : 8;
+  return G <= 2 ? 4 : 8;
 }
 // CTAs per SM the register budget is sized for (at most 12 warps of 170
 // registers per SM)

@@ -75,14 +75,14 @@ constexpr int kAttnMinStagesPerWarp = 4;
 // ceil(NS / (warps * kAttnChunksPerWarp)) stages or more, so at most
 // warps * kAttnChunksPerWarp of them.
 // Unit split (one cluster of C CTAs per (sequence, kv head) unit, merged on
-// chip) instead of a static stream-K split when, with the largest C >= 2 at
-// which every cluster is resident at once, it runs at least this share of
-// the stream-K grid's warps.  Its merge costs a fraction of stream-K's
-// cross-SM one, so it wins even on fewer SMs: on the paper's model shape (48
-// units; clusters of 3 do not all fit) 96 SMs of 12 warps took 10.9 us per
-// launch against 17.4 us for stream-K on all 152.  It is static, so it
-// suits units of similar length, which the small launches of one decode
-// step have.
+// chip) instead of a static stream-K split when, with the largest C at which
+// every cluster is resident at once, it runs at least this share of the
+// stream-K grid's warps.  Its merge costs a fraction of stream-K's cross-SM
+// one, so it wins even with fewer warps: measured side by side, 10.5 vs 17.4
+// us per launch on the paper's model shape (48 units, clusters of 8 CTAs of
+// 4 warps) and 17.4 vs 20.2 us on 192 units of 2048 tokens (C = 1, 768
+// warps against 1216).  It is static, so it suits units of similar length,
+// which the small launches of one decode step have.
 constexpr double kAttnUnitMinWarpShare = 0.6;
 
 // Resident clusters of C unit-split CTAs for (dtype, d, G) on this device,
@@ -160,7 +160,7 @@ AttnPlan attn_plan(const wm_config& c, int32_t B, int32_t max_pages, uint32_t fl
     int64_t C = nsm / units;
     pl.unit_ctas = (int)(C < 1 ? 1 : C > wm::kAttnUnitMaxCluster ? wm::kAttnUnitMaxCluster : C);
   } else if (!force_dynamic && pl.chunk_stages == 0 && unit_warps > 0) {
-    for (int C = wm::kAttnUnitMaxCluster; C >= 2; --C) {
+    for (int C = wm::kAttnUnitMaxCluster; C >= 1; --C) {
       if (unit_max_clusters(c.dtype, c.d, G, C) < units) continue;
       if ((double)(units * C * unit_warps) >= kAttnUnitMinWarpShare * pl.nwarps) pl.unit_ctas = C;
       break;

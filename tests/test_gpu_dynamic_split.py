@@ -1,5 +1,5 @@
-"""Decode attention on the dynamic split (Sec. 3.1 Step 3, dummy of Sec. 3.2),
-every output row against the fp64 oracle.
+"""Decode attention on the stream-K kernel's splits (Sec. 3.1 Step 3, dummy of
+Sec. 3.2), every output row against the fp64 oracle.
 
 Launches reading 2 GB of K/V or more cut the KV stream into about eight
 chunks per warp and hand them out from a device counter; units crossing
@@ -87,4 +87,55 @@ def test_dynamic_split_repeated_launches_leave_no_stale_state():
         torch.cuda.synchronize()
         assert H.rel_err(H.to_f64(out), want[:B]) <= H.TOL[w.dtype], B
     assert sess.read_status() == 0
+    _free()
+
+
+def test_static_split_of_many_short_units_every_row():
+    """More units than resident unit-split clusters (768 units of up to 512
+    tokens, 50 MB): the default plan streams with the static split, one chunk
+    per warp, units crossing chunk ends merged from partial records."""
+    w = configs.get("no_compression").with_(B=64, L=2, k=2, ctx=512, ctx_lo=1, permute_pages=True)
+    prob, sess, dp = H.setup(w)
+    plan = W.wm_decode_attn_plan(sess.cfg, w.B, prob.max_pages)
+    assert plan["unit_ctas"] == 0 and plan["chunk_stages"] == 0, plan
+    for layer in range(w.L):
+        got = _run(sess, dp, layer, False)
+        torch.cuda.synchronize()
+        err = H.rel_err(H.to_f64(got), H.oracle_attn_full(prob, layer))
+        assert err <= H.TOL[w.dtype], (layer, err)
+    assert sess.read_status() == 0
+    _free()
+
+
+def test_stream_k_edge_cases():
+    """On the counter-driven split: slots past the length never reach the
+    output, a dummy-only sequence returns the dummy's value, a bad page id or
+    length sets WM_ERR_BOUNDS and a bad length zero-fills its rows."""
+    w = configs.get("no_compression").with_(B=4, L=1, k=1)
+    lens = [37, 16, 1000, 1]
+    prob, sess, dp = H.setup(w, seq_lens=lens)
+    base = _run(sess, dp, 0, True).clone()
+    torch.cuda.synchronize()
+    assert H.rel_err(H.to_f64(base), H.oracle_attn_full(prob, 0)) <= H.TOL[w.dtype]
+    pg = int(prob.page_table[3, 0])
+    assert torch.equal(base[3], sess.v_pool[0, pg, :, 0, :])
+    for b, S in enumerate(lens):
+        for i in range(int((prob.page_table[b] >= 0).sum())):
+            lo = max(0, S - i * w.page)
+            if lo < w.page:
+                p = int(prob.page_table[b, i])
+                sess.k_pool[:, p, :, lo:, :] = float("nan")
+                sess.v_pool[:, p, :, lo:, :] = float("nan")
+    assert torch.equal(_run(sess, dp, 0, True), base)
+    assert sess.read_status() == 0
+    dp.page_table[2, 3] = prob.num_pages + 5
+    _run(sess, dp, 0, True)
+    torch.cuda.synchronize()
+    assert sess.read_status() == 4  # WM_ERR_BOUNDS
+    dp.page_table[2, 3] = int(prob.page_table[2, 3])
+    dp.seq_lens[1] = 0
+    out = _run(sess, dp, 0, True)
+    torch.cuda.synchronize()
+    assert sess.read_status() == 4
+    assert torch.count_nonzero(out[1].float()) == 0
     _free()

@@ -254,20 +254,22 @@ def test_inputs_ready_chain_matches_default_launches(name, overrides):
     _free()
 
 
-def test_graph_replay_over_changing_lengths():
+@pytest.mark.parametrize("dynamic", [False, True])
+def test_graph_replay_over_changing_lengths(dynamic):
     """A decode loop replays one captured launch while the lengths change
-    underneath it (the replay keeps the call's epoch): the chunk layout moves
-    with the lengths, and no flag or ticket left by an earlier replay passes
-    for this replay's records."""
+    underneath it (the replay keeps the call's epoch): on the counter-driven
+    split the chunk layout moves with the lengths, and no flag or ticket left
+    by an earlier replay passes for this replay's records; the default plan
+    here is the unit split."""
     w = configs.get("no_compression").with_(L=2, k=2)
     prob, sess, dp = H.setup(w)
     lens = dp.seq_lens.clone()
     out = torch.empty((w.B, w.Hq, w.d), dtype=sess.dtype, device=sess.device)
-    sess.decode_attn(0, dp.q[0], dp.page_table, lens, out)  # warm-up outside capture
+    sess.decode_attn(0, dp.q[0], dp.page_table, lens, out, dynamic_split=dynamic)  # warm-up
     torch.cuda.synchronize()
     g = torch.cuda.CUDAGraph()
     with torch.cuda.graph(g):
-        sess.decode_attn(0, dp.q[0], dp.page_table, lens, out)
+        sess.decode_attn(0, dp.q[0], dp.page_table, lens, out, dynamic_split=dynamic)
     rng = np.random.default_rng(3)
     full = np.asarray(prob.seq_lens, np.int64)
     sets = [full, np.maximum(1, full // 3), rng.integers(1, full + 1), full - 17,
@@ -289,14 +291,16 @@ def test_graph_replay_over_changing_lengths():
 
 def test_workspace_reused_across_batch_sizes():
     """One workspace serves calls whose plans lay partial records out
-    differently (a smaller batch splits into fewer chunks): words left by
+    differently (a smaller batch splits into fewer chunks), mixed with calls
+    on the unit split, which leaves the workspace alone: words left by
     another call never pass for published records."""
     w = configs.get("no_compression").with_(L=2, k=2)
     prob, sess, dp = H.setup(w)
     want = H.oracle_attn_full(prob, 0)
-    for B in (w.B, 5, 11, w.B):
+    for B, dyn in ((w.B, True), (5, True), (11, False), (w.B, True), (3, False), (7, True)):
         out = torch.full((B, w.Hq, w.d), float("nan"), dtype=sess.dtype, device=sess.device)
-        sess.decode_attn(0, dp.q[0][:B], dp.page_table[:B], dp.seq_lens[:B], out, B=B)
+        sess.decode_attn(0, dp.q[0][:B], dp.page_table[:B], dp.seq_lens[:B], out, B=B,
+                         dynamic_split=dyn)
         torch.cuda.synchronize()
         err = H.rel_err(H.to_f64(out), want[:B])
         assert err <= H.TOL[w.dtype], (B, err)

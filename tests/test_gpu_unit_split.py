@@ -47,6 +47,7 @@ def _plan(sess, w, prob, flags=W.WM_ATTN_UNIT_SPLIT):
     ("no_compression", dict(), None, 1),                             # 192 units > SMs: C = 1
     ("no_compression", dict(L=3, k=2, permute_pages=True), RAGGED16, 1),
     ("paper_k16", dict(L=4, k=4), None, 3),                          # 6/3 heads of 96
+    ("paper_k16", dict(L=2, k=2, B=5), [2048, 7, 1, 1000, 2049], 8),
     ("paper_k16", dict(L=2, k=2, permute_pages=True), RAGGED16, 3),
     ("compress50", dict(B=8, L=2, k=2, Hq=64, Hkv=8),                # G = 8, 64 units
      [4096, 3000, 129, 2, 4096, 4096, 4000, 3500], 2),
@@ -125,18 +126,17 @@ def test_unit_split_edge_cases(name):
 
 
 def test_default_plan_takes_the_unit_split_only_where_it_keeps_the_warps():
-    """Small launches whose units fit resident clusters of >= 2 CTAs with at
-    least 60% of the static grid's warps take the unit split; launches with
-    more units than that, and launches of 2 GB or more, stream."""
-    nsm = torch.cuda.get_device_properties(0).multi_processor_count
+    """Small launches whose units fit resident clusters with at least 60% of
+    the static grid's warps take the unit split; launches with more units
+    than that, and launches of 2 GB or more, stream."""
     for name, unit in (("paper_k16", True), ("paper_k1", True), ("tiny_f32", True),
-                       ("no_compression", False), ("compress50", False), ("large", False),
+                       ("no_compression", True), ("compress50", False), ("large", False),
                        ("long32k", False)):
         w = configs.get(name)
         c = H.config_of(w)
         max_pages = -(-(w.ctx + 1) // w.page)
         plan = W.wm_decode_attn_plan(c, w.B, max_pages)
-        assert (plan["unit_ctas"] >= 2) == unit, (name, plan)
+        assert (plan["unit_ctas"] >= 1) == unit, (name, plan)
         if unit:
             static = W.wm_decode_attn_plan(c, w.B, max_pages, W.WM_ATTN_DYNAMIC_SPLIT)
             assert plan["grid"] == w.B * w.Hkv * plan["unit_ctas"], (name, plan)

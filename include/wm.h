@@ -231,10 +231,11 @@ wm_status wm_decode_attn(const wm_config* cfg, const wm_cache* cache, int32_t la
  *     C = min(8, max(1, SMs / units)) CTAs whose warps each stream an equal
  *     share of the unit and merge on chip (shared and distributed shared
  *     memory), whatever the launch size.  Without it the split is taken only
- *     for launches below 2 GB where, at the largest C whose clusters are all
- *     resident at once, it runs at least 60% of the warps of the static
- *     split above (the paper's model shape, 48 units: C = 8; 192 units:
- *     C = 1); every other launch streams as above.  The unit split uses no
+ *     for launches below 2 GB, or of a single sequence, where, at the
+ *     largest C whose clusters are all resident at once, it runs at least
+ *     60% of the warps of the static split above (the paper's model shape,
+ *     48 units: C = 8; 192 units: C = 1; one sequence of 32 heads: C = 8);
+ *     every other launch streams as above.  The unit split uses no
  *     workspace and gives the same result within rounding.
  * Unknown flag bits, or DYNAMIC_SPLIT together with UNIT_SPLIT, return
  * WM_ERR_INVALID_ARG.

@@ -82,7 +82,11 @@ constexpr int kAttnMinStagesPerWarp = 4;
 // us per launch on the paper's model shape (48 units, clusters of 8 CTAs of
 // 4 warps) and 17.4 vs 20.2 us on 192 units of 2048 tokens (C = 1, 768
 // warps against 1216).  It is static, so it suits units of similar length,
-// which the small launches of one decode step have.
+// which the small launches of one decode step have.  Launches of 2 GB or
+// more take it only for a single sequence, whose units all have the same
+// length (one sequence of 131072 slots, 32 units in clusters of 8: 317 vs
+// 357 us per launch on stream-K); with more sequences the lengths may differ
+// and stream-K balances them.
 constexpr double kAttnUnitMinWarpShare = 0.6;
 
 // Resident clusters of C unit-split CTAs for (dtype, d, G) on this device,
@@ -159,7 +163,7 @@ AttnPlan attn_plan(const wm_config& c, int32_t B, int32_t max_pages, uint32_t fl
   if (force_unit) {
     int64_t C = nsm / units;
     pl.unit_ctas = (int)(C < 1 ? 1 : C > wm::kAttnUnitMaxCluster ? wm::kAttnUnitMaxCluster : C);
-  } else if (!force_dynamic && pl.chunk_stages == 0 && unit_warps > 0) {
+  } else if (!force_dynamic && (pl.chunk_stages == 0 || B == 1) && unit_warps > 0) {
     for (int C = wm::kAttnUnitMaxCluster; C >= 1; --C) {
       if (unit_max_clusters(c.dtype, c.d, G, C) < units) continue;
       if ((double)(units * C * unit_warps) >= kAttnUnitMinWarpShare * pl.nwarps) pl.unit_ctas = C;

@@ -1,8 +1,9 @@
 """The full-size workloads, every output against the fp64 oracle.
 
 Decode attention (Sec. 3.1 Step 3, dummy of Sec. 3.2): one whole layer of
-each of the four full-size workloads -- 1.1 GB (static split) to 17.2 GB (the
-counter-driven split) of K/V per launch -- every (sequence, query head) row.
+each of the full-size workloads -- 1.1 GB (static split) to 17.2 GB (the
+counter-driven split) of K/V per launch, and one sequence of 131072 slots
+(2.15 GB, the unit split) -- every (sequence, query head) row.
 The pool (Sec. 3.1 Steps 1-2, appended as in Sec. 3.2): every token and
 every channel of the key and value rows written.  The host regenerates only
 what each comparison reads, a sequence's pages of one channel at a time.
@@ -29,14 +30,20 @@ def _free():
     torch.cuda.empty_cache()
 
 
-@pytest.mark.parametrize("name,layer", [("compress50", 5), ("large", 13), ("long32k", 0),
-                                        ("long64k", 7), ("long128k", 5)])
-def test_full_size_layer_every_row(name, layer):
-    w = configs.get(name)
+@pytest.mark.parametrize("name,layer,overrides", [
+    ("compress50", 5, {}), ("large", 13, {}), ("long32k", 0, {}), ("long64k", 7, {}),
+    ("long128k", 5, {}),
+    ("long128k", 9, dict(B=1, k=2)),  # one sequence of 2.15 GB: the unit split, clusters of 8
+])
+def test_full_size_layer_every_row(name, layer, overrides):
+    w = configs.get(name).with_(**overrides)
     prob, sess, dp = H.setup(w)
     plan = W.wm_decode_attn_plan(sess.cfg, w.B, prob.max_pages)
     kv_bytes = float(w.B) * w.Hkv * prob.max_pages * w.page * 2 * w.d * w.elem_bytes
-    assert (plan["chunk_stages"] > 0) == (kv_bytes >= DYNAMIC_BYTES), plan
+    if w.B == 1:
+        assert plan["unit_ctas"] >= 2 and plan["chunk_stages"] == 0, plan
+    else:
+        assert (plan["chunk_stages"] > 0) == (kv_bytes >= DYNAMIC_BYTES), plan
     out = H.run_attn(sess, dp, layer)
     torch.cuda.synchronize()
     assert sess.read_status() == 0

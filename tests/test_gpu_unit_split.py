@@ -126,13 +126,16 @@ def test_unit_split_edge_cases(name):
 
 
 def test_default_plan_takes_the_unit_split_only_where_it_keeps_the_warps():
-    """Small launches whose units fit resident clusters with at least 60% of
-    the static grid's warps take the unit split; launches with more units
-    than that, and launches of 2 GB or more, stream."""
-    for name, unit in (("paper_k16", True), ("paper_k1", True), ("tiny_f32", True),
-                       ("no_compression", True), ("compress50", False), ("large", False),
-                       ("long32k", False)):
-        w = configs.get(name)
+    """Launches below 2 GB, or of one sequence, whose units fit resident
+    clusters with at least 60% of the static grid's warps take the unit
+    split; launches with more units than that, and launches of 2 GB or more
+    over several sequences, stream."""
+    for name, over, unit in (("paper_k16", {}, True), ("paper_k1", {}, True),
+                             ("tiny_f32", {}, True), ("no_compression", {}, True),
+                             ("compress50", {}, False), ("large", {}, False),
+                             ("long32k", {}, False), ("long128k", {}, False),
+                             ("long128k", dict(B=1), True), ("long128k", dict(B=2), False)):
+        w = configs.get(name).with_(**over)
         c = H.config_of(w)
         max_pages = -(-(w.ctx + 1) // w.page)
         plan = W.wm_decode_attn_plan(c, w.B, max_pages)

@@ -15,7 +15,8 @@
 // waited on; the stream-K kernel's cross-SM merge (flags raised on other SMs,
 // records landed from L2) sits on the critical path of such short launches.
 // The split is static, so it suits launches whose units have similar lengths;
-// the planner takes it only when C x units fills nearly every SM.
+// the planner takes it for launches below 2 GB, or of one sequence, when all
+// its clusters are resident at once with enough warps (csrc/wm_api.cu).
 #include <cooperative_groups.h>
 
 #include "attn_kernel.cuh"

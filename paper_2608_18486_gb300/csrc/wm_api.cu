@@ -265,7 +265,8 @@ wm_status decode_attn_impl(const wm_config* c, const wm_cache* cache, int32_t la
   p.inputs_ready = (flags & WM_ATTN_INPUTS_READY) ? 1 : 0;
   p.epoch = next_attn_epoch();
   p.qscale = (float)(1.4426950408889634 / sqrt((double)c->d));
-  if (clear_workspace &&
+  // (the unit split touches no workspace)
+  if (clear_workspace && pl.unit_ctas == 0 &&
       cudaMemsetAsync(workspace, 0, pl.total, (cudaStream_t)stream) != cudaSuccess)
     return WM_ERR_CUDA;
   cudaError_t e =

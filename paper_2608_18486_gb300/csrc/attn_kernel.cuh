@@ -852,13 +852,9 @@ __global__ void __launch_bounds__(kThreads, attn_ctas_per_sm(SB, G)) decode_attn
 
 template <typename T, int HD, int G, int SB>
 inline cudaError_t launch_t(const AttnParams& p, int grid, size_t smem, cudaStream_t stream) {
-  static size_t smem_set = 0;  // largest dynamic smem opted into so far
+  static size_t smem_set[kSmemOptDevices] = {};
   auto kern = decode_attn_kernel<T, HD, G, SB>;
-  if (smem > smem_set) {
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    smem_set = smem;
-  }
+  if (cudaError_t e = opt_in_smem(kern, smem, smem_set); e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(grid);
   cfg.blockDim = dim3(kThreads);

@@ -350,13 +350,9 @@ __global__ void __launch_bounds__(unit_warps<T, HD, G, SB>() * 32,
 template <typename T, int HD, int G, int SB>
 inline cudaError_t launch_unit_t(const AttnParams& p, int units, int cluster, size_t smem,
                                  cudaStream_t stream) {
-  static size_t smem_set = 0;  // largest dynamic smem opted into so far
+  static size_t smem_set[kSmemOptDevices] = {};
   auto kern = decode_attn_unit_kernel<T, HD, G, SB>;
-  if (smem > smem_set) {
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    smem_set = smem;
-  }
+  if (cudaError_t e = opt_in_smem(kern, smem, smem_set); e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)units * (unsigned)cluster);
   cfg.blockDim = dim3(unit_warps<T, HD, G, SB>() * 32);

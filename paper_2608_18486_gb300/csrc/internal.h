@@ -8,6 +8,21 @@
 
 namespace wm {
 
+// Opt kernel `kern` into `smem` bytes of dynamic shared memory on the current
+// device (the limit is a per-device attribute of the function).  `done`
+// holds, per device, the largest value set so far.
+constexpr int kSmemOptDevices = 64;
+template <typename Kern>
+inline cudaError_t opt_in_smem(Kern kern, size_t smem, size_t (&done)[kSmemOptDevices]) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return cudaErrorInvalidDevice;
+  const bool cached = dev >= 0 && dev < kSmemOptDevices;
+  if (cached && smem <= done[dev]) return cudaSuccess;
+  const cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e == cudaSuccess && cached) done[dev] = smem;
+  return e;
+}
+
 // ------------------------------------------------------------ attention
 struct AttnParams {
   const void* k_pool;     // channel c(layer) base of the K pool

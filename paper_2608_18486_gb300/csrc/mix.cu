@@ -701,12 +701,9 @@ cudaError_t launch_all(MixParams& p, cudaStream_t s) {
                         16 + (size_t)lc * per_layer;
     dim3 grid((p.B + tb - 1) / tb, 2, (p.k + kMixCG - 1) / kMixCG);
     auto kern = two ? mix_tokens_kernel<T, 2> : mix_tokens_kernel<T, 1>;
-    static size_t smem_set[2] = {0, 0};  // largest dynamic smem opted into, per variant
-    if (smem > smem_set[two]) {
-      e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-      if (e != cudaSuccess) return e;
-      smem_set[two] = smem;
-    }
+    static size_t smem_set[2][kSmemOptDevices] = {};  // per variant and device
+    e = opt_in_smem(kern, smem, smem_set[two]);
+    if (e != cudaSuccess) return e;
     e = launch_pdl(kern, grid, dim3(tb * tpt), smem, s, p, tpt, tb, lc);
     if (e != cudaSuccess) return e;
   } else {

@@ -461,14 +461,10 @@ __global__ void __launch_bounds__(kPThreads, 1)
 template <int HD>
 cudaError_t launch_hd(const CUtensorMap& q, const CUtensorMap& k, const CUtensorMap& v,
                       const PrefillParams& p, cudaStream_t s) {
-  static bool attr_set = false;
+  static size_t smem_set[kSmemOptDevices] = {};
   auto kern = prefill_attn_kernel<HD>;
-  if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)PShape<HD>::SMEM);
-    if (e != cudaSuccess) return e;
-    attr_set = true;
-  }
+  if (cudaError_t e = opt_in_smem(kern, (size_t)PShape<HD>::SMEM, smem_set); e != cudaSuccess)
+    return e;
   cudaLaunchConfig_t cfg = {};
   const int rows_cta = p.pair ? kPM : kQT * kPM;
   cfg.gridDim = dim3((p.Tq + rows_cta - 1) / rows_cta, p.pair ? p.Hq / kQT : p.Hq, p.B);

@@ -261,13 +261,9 @@ size_t tc_smem(int stages, int BN) {
 template <int HD, int MODE>
 cudaError_t launch_mode(dim3 grid, size_t smem, const CUtensorMap& w0, const CUtensorMap& w1,
                         const CUtensorMap& x, const ProjTcParams& p, cudaStream_t s) {
-  static size_t smem_set = 0;
+  static size_t smem_set[kSmemOptDevices] = {};
   auto kern = proj_tc_kernel<HD, MODE>;
-  if (smem > smem_set) {
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    smem_set = smem;
-  }
+  if (cudaError_t e = opt_in_smem(kern, smem, smem_set); e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = grid;
   cfg.blockDim = dim3(kTcThreads);
